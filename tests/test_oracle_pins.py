@@ -1,0 +1,411 @@
+"""Pins of the fp64 oracle against facts fixed by the paper and by mathematics.
+
+Each test checks the oracle against something other than itself: hand-derived
+examples (tests/golden), closed forms, an independent formulation (complex
+rotation, a library softmax, exact rational arithmetic), invariants the method
+states (§4.1-§4.2, Eqs. 2-3) or brute force on tiny inputs.
+"""
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+from scipy.special import softmax
+
+from oracle import kvm_oracle as O
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+rng = np.random.default_rng(1234)
+
+
+def _gold(name):
+    with open(os.path.join(GOLD, name)) as f:
+        return json.load(f)
+
+
+def _unit(x):
+    return x / np.linalg.norm(x, axis=-1, keepdims=True)
+
+
+# ---------------------------------------------------------------- golden
+def test_golden_gdn_hand_example():
+    g = _gold("gdn_hand_2d.json")
+    q = np.array(g["q"])[:, None, :]
+    k = np.array(g["k"])[:, None, :]
+    v = np.array(g["v"])[:, None, :]
+    a = np.array(g["alpha"])[:, None]
+    b = np.array(g["beta"])[:, None]
+    S0 = np.array(g["S0"])[None]
+    o, S = O.gdn_recurrent(q, k, v, a, b, S0)
+    np.testing.assert_allclose(o[:, 0], g["o"], atol=1e-12)
+    np.testing.assert_allclose(S[0], g["S"], atol=1e-12)
+
+
+def test_golden_attention_hand_example():
+    g = _gold("attn_hand.json")
+    cache = O.AttnCache(np.array(g["cache_k"]), np.array(g["cache_v"]), np.array(g["cache_pos"]))
+    out, new = O.tail_attn_prefill(cache, np.array(g["q"]), np.array(g["k_new"]),
+                                   np.array(g["v_new"]), g["cursor"], 0, 1e4)
+    np.testing.assert_allclose(out, g["out"], atol=1e-12)
+    assert list(new.pos) == [0, g["cursor"]]
+
+
+def test_golden_rope_hand_example():
+    g = _gold("rope_hand.json")
+    x = np.array(g["x"], dtype=np.float64)[:, None, :]
+    pos = np.full(x.shape[0], g["pos"])
+    out = O.rope(x, pos, g["R"], g["theta"])
+    np.testing.assert_allclose(out[:, 0], g["out"], atol=1e-12)
+
+
+# ---------------------------------------------------------------- RoPE
+def test_rope_matches_complex_rotation():
+    """RoFormer's complex form: z_d = x_d + i x_{d+R/2} times exp(i pos w_d)."""
+    D, R, theta = 16, 8, 1e4
+    x = rng.standard_normal((5, 3, D))
+    pos = np.array([0, 1, 17, 4096, 479547])
+    out = O.rope(x, pos, R, theta)
+    h = R // 2
+    for n in range(5):
+        for d in range(h):
+            w = theta ** (-(2 * d) / R)
+            z = complex(x[n, 0, d], x[n, 0, d + h]) * complex(math.cos(pos[n] * w), math.sin(pos[n] * w))
+            assert abs(out[n, 0, d] - z.real) < 1e-9
+            assert abs(out[n, 0, d + h] - z.imag) < 1e-9
+    np.testing.assert_array_equal(out[:, :, R:], x[:, :, R:])
+
+
+def test_rope_relative_position_and_norm():
+    D, R, theta = 64, 64, 1e4
+    q = rng.standard_normal((1, 1, D))
+    k = rng.standard_normal((1, 1, D))
+    for m, n, delta in [(10, 3, 1000), (5, 5, 123456), (0, 40, 400000)]:
+        a = O.rope(q, [m], R, theta)[0, 0] @ O.rope(k, [n], R, theta)[0, 0]
+        b = O.rope(q, [m + delta], R, theta)[0, 0] @ O.rope(k, [n + delta], R, theta)[0, 0]
+        assert abs(a - b) < 1e-8 * max(1.0, abs(a))
+    r = O.rope(q, [479547], R, theta)
+    assert abs(np.linalg.norm(r) - np.linalg.norm(q)) < 1e-12
+    np.testing.assert_array_equal(O.rope(q, [0], R, theta), q)
+
+
+def test_rope_frequency_values():
+    w = O.rope_frequencies(64, 1e4)
+    assert w[0] == 1.0
+    assert abs(w[1] - 10 ** (-0.125)) < 1e-15
+    assert abs(w[31] - 1e4 ** (-62 / 64)) < 1e-18
+
+
+# ---------------------------------------------------------------- attention
+def test_attention_single_key_returns_value():
+    cache = O.AttnCache(np.zeros((2, 0, 8)), np.zeros((2, 0, 8)), np.zeros(0))
+    q = rng.standard_normal((1, 4, 8))
+    k = rng.standard_normal((1, 2, 8))
+    v = rng.standard_normal((1, 2, 8))
+    out, _ = O.tail_attn_prefill(cache, q, k, v, 7, 8, 1e4)
+    for h in range(4):
+        np.testing.assert_allclose(out[0, h], v[0, h // 2], atol=1e-14)
+
+
+def test_attention_constant_values_weights_sum_to_one():
+    L, M, D = 9, 3, 8
+    cache = O.AttnCache(rng.standard_normal((1, L, D)), np.ones((1, L, D)) * 2.5, np.arange(L))
+    out, _ = O.tail_attn_prefill(cache, rng.standard_normal((M, 2, D)), rng.standard_normal((M, 1, D)),
+                                 np.ones((M, 1, D)) * 2.5, L, 4, 1e4)
+    np.testing.assert_allclose(out, 2.5, atol=1e-13)
+
+
+def _masked_reference(cache_full, keep, q, k_new, v_new, p, R, theta):
+    """Library softmax over the UNcompacted cache with removed keys at -inf."""
+    M, Hq, D = q.shape
+    Hkv = cache_full.K.shape[0]
+    g = Hq // Hkv
+    pos_new = p + np.arange(M)
+    qr = O.rope(q, pos_new, R, theta)
+    kr = O.rope(k_new, pos_new, R, theta)
+    out = np.zeros_like(qr)
+    L = cache_full.K.shape[1]
+    for i in range(M):
+        for h in range(Hq):
+            keys = np.concatenate([cache_full.K[h // g], kr[:, h // g]])
+            vals = np.concatenate([cache_full.V[h // g], v_new[:, h // g]])
+            allow = np.concatenate([keep, np.arange(M) <= i])
+            s = np.where(allow, keys @ qr[i, h] / math.sqrt(D), -np.inf)
+            out[i, h] = softmax(s) @ vals
+    return out
+
+
+def test_removed_equals_masked():
+    """Eq. 2: attention over the compacted cache equals attention over the
+    full cache with the removed entries masked out."""
+    L, M, D, Hq, Hkv, R = 40, 5, 16, 4, 2, 8
+    full = O.AttnCache(rng.standard_normal((Hkv, L, D)), rng.standard_normal((Hkv, L, D)), np.arange(L))
+    begins, ends = [3, 20], [7, 31]
+    K, V, pos, _ = O.kv_compact(full.K, full.V, full.pos, begins, ends)
+    q = rng.standard_normal((M, Hq, D))
+    kn = rng.standard_normal((M, Hkv, D))
+    vn = rng.standard_normal((M, Hkv, D))
+    out, _ = O.tail_attn_prefill(O.AttnCache(K, V, pos), q, kn, vn, 50, R, 1e4)
+    ref = _masked_reference(full, O.keep_mask(L, begins, ends), q, kn, vn, 50, R, 1e4)
+    np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_gqa_equals_mha_with_replicated_kv():
+    L, M, D, Hq, Hkv, R = 12, 4, 8, 4, 2, 8
+    K = rng.standard_normal((Hkv, L, D))
+    V = rng.standard_normal((Hkv, L, D))
+    q = rng.standard_normal((M, Hq, D))
+    kn = rng.standard_normal((M, Hkv, D))
+    vn = rng.standard_normal((M, Hkv, D))
+    out, _ = O.tail_attn_prefill(O.AttnCache(K, V, np.arange(L)), q, kn, vn, L, R, 1e4)
+    rep = [0, 0, 1, 1]
+    out2, _ = O.tail_attn_prefill(O.AttnCache(K[rep], V[rep], np.arange(L)), q, kn[:, rep], vn[:, rep],
+                                  L, R, 1e4)
+    np.testing.assert_allclose(out, out2, atol=1e-13)
+
+
+def test_attention_brute_force_tiny():
+    """Scalar brute force: complex-form rotation and an explicit softmax."""
+    D, R, theta, L, M = 4, 2, 10.0, 3, 2
+    Kc = rng.standard_normal((1, L, D))
+    Vc = rng.standard_normal((1, L, D))
+    q = rng.standard_normal((M, 1, D))
+    kn = rng.standard_normal((M, 1, D))
+    vn = rng.standard_normal((M, 1, D))
+    p = 11
+    out, _ = O.tail_attn_prefill(O.AttnCache(Kc, Vc, np.arange(L)), q, kn, vn, p, R, theta)
+
+    def rot(x, pos):
+        z = complex(x[0], x[1]) * complex(math.cos(pos), math.sin(pos))   # R = 2: w_0 = 1
+        return [z.real, z.imag, x[2], x[3]]
+
+    for i in range(M):
+        qi = rot(q[i, 0], p + i)
+        keys = [list(Kc[0, j]) for j in range(L)] + [rot(kn[j, 0], p + j) for j in range(i + 1)]
+        vals = [list(Vc[0, j]) for j in range(L)] + [list(vn[j, 0]) for j in range(i + 1)]
+        sc = [sum(a * b for a, b in zip(qi, kk)) / 2.0 for kk in keys]
+        ws = [math.exp(s) for s in sc]
+        tot = sum(ws)
+        for d in range(D):
+            ref = sum(w * vv[d] for w, vv in zip(ws, vals)) / tot
+            assert abs(out[i, 0, d] - ref) < 1e-12
+
+
+def test_attention_relative_shift_invariance():
+    """Shifting every position by the same amount leaves the outputs alone."""
+    D, R, Hq, Hkv = 16, 16, 2, 1
+    toks = {"q": rng.standard_normal((10, Hq, D)), "k": rng.standard_normal((10, Hkv, D)),
+            "v": rng.standard_normal((10, Hkv, D))}
+    empty = O.AttnCache(np.zeros((Hkv, 0, D)), np.zeros((Hkv, 0, D)), np.zeros(0))
+    a, _ = O.tail_attn_prefill(empty, toks["q"], toks["k"], toks["v"], 0, R, 1e4)
+    b, cb = O.tail_attn_prefill(empty, toks["q"], toks["k"], toks["v"], 250000, R, 1e4)
+    np.testing.assert_allclose(a, b, atol=1e-9)
+    assert list(cb.pos) == list(range(250000, 250010))
+
+
+# ---------------------------------------------------------------- delta rule
+def _gdn_inputs(M, H, dk, dv, unit=True):
+    k = rng.standard_normal((M, H, dk))
+    if unit:
+        k = _unit(k)
+    return (rng.standard_normal((M, H, dk)), k, rng.standard_normal((M, H, dv)),
+            1 / (1 + np.exp(-rng.normal(3, 0.5, (M, H)))), 1 / (1 + np.exp(-rng.standard_normal((M, H)))),
+            rng.standard_normal((H, dv, dk)) * 0.2)
+
+
+def test_gdn_identity_gates_keep_state():
+    q, k, v, a, b, S0 = _gdn_inputs(7, 2, 4, 3)
+    o, S = O.gdn_recurrent(q, k, v, np.ones_like(a), np.zeros_like(b), S0)
+    np.testing.assert_allclose(S, S0, atol=1e-15)
+    np.testing.assert_allclose(o, np.einsum("hvk,thk->thv", S0, q), atol=1e-13)
+
+
+def test_gdn_unit_key_recall():
+    """alpha = beta = 1 and |k| = 1: the delta rule stores v exactly, S_t k_t = v_t."""
+    q, k, v, a, b, S0 = _gdn_inputs(6, 3, 8, 5)
+    M = k.shape[0]
+    for t in range(1, M + 1):
+        _, S = O.gdn_recurrent(q[:t], k[:t], v[:t], np.ones_like(a[:t]), np.ones_like(b[:t]), S0)
+        for h in range(3):
+            np.testing.assert_allclose(S[h] @ k[t - 1, h], v[t - 1, h], atol=1e-12)
+
+
+def test_gdn_general_key_identity():
+    """S_t k_t = alpha (1 - beta |k|^2) S_{t-1} k_t + beta |k|^2 v_t for any k."""
+    q, k, v, a, b, S0 = _gdn_inputs(5, 2, 6, 4, unit=False)
+    Sp = S0
+    for t in range(5):
+        _, S = O.gdn_recurrent(q[t:t + 1], k[t:t + 1], v[t:t + 1], a[t:t + 1], b[t:t + 1], Sp)
+        for h in range(2):
+            kk = k[t, h] @ k[t, h]
+            ref = a[t, h] * (1 - b[t, h] * kk) * (Sp[h] @ k[t, h]) + b[t, h] * kk * v[t, h]
+            np.testing.assert_allclose(S[h] @ k[t, h], ref, atol=1e-11)
+        Sp = S
+
+
+def test_gdn_orthonormal_keys_closed_form():
+    """Orthonormal keys never interfere: S_n = sum_j (prod_{u>j} alpha_u) beta_j v_j k_j^T."""
+    d = 6
+    Qm, _ = np.linalg.qr(rng.standard_normal((d, d)))
+    k = Qm.T[:, None, :]                       # d tokens, 1 head
+    v = rng.standard_normal((d, 1, 3))
+    a = rng.uniform(0.5, 1.0, (d, 1))
+    b = rng.uniform(0.1, 1.0, (d, 1))
+    _, S = O.gdn_recurrent(rng.standard_normal((d, 1, d)), k, v, a, b, np.zeros((1, 3, d)))
+    ref = np.zeros((3, d))
+    for j in range(d):
+        ref += np.prod(a[j + 1:, 0]) * b[j, 0] * np.outer(v[j, 0], k[j, 0])
+    np.testing.assert_allclose(S[0], ref, atol=1e-13)
+
+
+def test_gdn_exact_rational_brute_force():
+    """Exact rational arithmetic (fractions) on a tiny 2x2 case, three tokens."""
+    toks = [((Fraction(1, 2), Fraction(1, 3)), (Fraction(3, 5), Fraction(4, 5)), (Fraction(1), Fraction(-2)),
+             Fraction(7, 8), Fraction(1, 4)),
+            ((Fraction(-1), Fraction(2)), (Fraction(1), Fraction(0)), (Fraction(1, 3), Fraction(1, 2)),
+             Fraction(3, 4), Fraction(2, 3)),
+            ((Fraction(2), Fraction(1)), (Fraction(5, 13), Fraction(12, 13)), (Fraction(-3, 2), Fraction(1)),
+             Fraction(9, 10), Fraction(1, 2))]
+    S = [[Fraction(1, 5), Fraction(-1, 2)], [Fraction(1, 3), Fraction(1)]]
+    S0 = np.array([[float(x) for x in r] for r in S])[None]
+    outs = []
+    for q, k, v, al, be in toks:
+        # S <- al*S*(I - be k k^T) + be v k^T, written entrywise
+        P = [[(1 if i == j else 0) - be * k[i] * k[j] for j in range(2)] for i in range(2)]
+        S = [[al * sum(S[r][m] * P[m][c] for m in range(2)) + be * v[r] * k[c] for c in range(2)]
+             for r in range(2)]
+        outs.append([sum(S[r][c] * q[c] for c in range(2)) for r in range(2)])
+    f = lambda i: np.array([[float(x) for x in t[i]] for t in toks])[:, None, :]
+    o, Sn = O.gdn_recurrent(f(0), f(1), f(2), np.array([[float(t[3])] for t in toks]),
+                            np.array([[float(t[4])] for t in toks]), S0)
+    np.testing.assert_allclose(o[:, 0], [[float(x) for x in r] for r in outs], atol=1e-14)
+    np.testing.assert_allclose(Sn[0], [[float(x) for x in r] for r in S], atol=1e-14)
+
+
+@pytest.mark.parametrize("M,C", [(150, 64), (64, 64), (1, 64), (37, 16), (200, 32)])
+def test_gdn_chunked_equals_recurrent(M, C):
+    q, k, v, a, b, S0 = _gdn_inputs(M, 3, 16, 12)
+    o1, S1 = O.gdn_recurrent(q, k, v, a, b, S0)
+    o2, S2 = O.gdn_chunked(q, k, v, a, b, S0, C)
+    np.testing.assert_allclose(o2, o1, atol=1e-11, rtol=1e-11)
+    np.testing.assert_allclose(S2, S1, atol=1e-11, rtol=1e-11)
+
+
+def test_gdn_resume_equals_uninterrupted():
+    """Continuing from a carried state equals running the whole sequence."""
+    q, k, v, a, b, S0 = _gdn_inputs(30, 2, 8, 8)
+    o, S = O.gdn_recurrent(q, k, v, a, b, S0)
+    o1, Sm = O.gdn_recurrent(q[:13], k[:13], v[:13], a[:13], b[:13], S0)
+    o2, S2 = O.gdn_recurrent(q[13:], k[13:], v[13:], a[13:], b[13:], Sm)
+    np.testing.assert_allclose(np.concatenate([o1, o2]), o, atol=1e-13)
+    np.testing.assert_allclose(S2, S, atol=1e-13)
+
+
+# ---------------------------------------------------------------- compaction
+def test_compact_counts_positions_order():
+    L = 100
+    K = rng.standard_normal((2, L, 4))
+    pos = np.arange(L) * 3 + 7
+    begins, ends = [0, 10, 50, 99], [2, 20, 51, 100]
+    K2, V2, p2, gather = O.kv_compact(K, K.copy(), pos, begins, ends)
+    assert K2.shape[1] == L - (2 + 10 + 1 + 1)
+    assert np.all(np.diff(p2) > 0)
+    np.testing.assert_array_equal(K2, K[:, gather])
+    removed = set().union(*[set(range(b, e)) for b, e in zip(begins, ends)])
+    assert list(gather) == [i for i in range(L) if i not in removed]
+
+
+def test_compact_identity_and_composition():
+    L = 60
+    K = rng.standard_normal((1, L, 2))
+    pos = np.arange(L)
+    K1, _, p1, g1 = O.kv_compact(K, K, pos, [], [])
+    np.testing.assert_array_equal(K1, K)
+    np.testing.assert_array_equal(g1, np.arange(L))
+    # two compactions in sequence == one compaction with the union of spans
+    Ka, _, pa, ga = O.kv_compact(K, K, pos, [5, 30], [10, 33])        # 52 left
+    Kb, _, pb, gb = O.kv_compact(Ka, Ka, pa, [0, 40], [3, 52])
+    Ku, _, pu, gu = O.kv_compact(K, K, pos, [0, 5, 30, 48], [3, 10, 33, 60])
+    np.testing.assert_array_equal(Kb, Ku)
+    np.testing.assert_array_equal(pb, pu)
+    np.testing.assert_array_equal(ga[gb], gu)
+
+
+@pytest.mark.parametrize("begins,ends", [([5, 3], [6, 4]), ([2, 4], [5, 7]), ([3], [3]), ([-1], [2]),
+                                         ([8], [11]), ([1, 2], [2])])
+def test_span_validation_rejects(begins, ends):
+    with pytest.raises(O.SpanError):
+        O.keep_mask(10, begins, ends)
+
+
+# ---------------------------------------------------------------- whole round
+def _stack():
+    return dict(layer_kind=[0, 1, 0, 1], Hkv=2, D=16, H=2, dk=8, dv=6, R=8, theta=1e4)
+
+
+def _tokens(n, st):
+    ins = {}
+    for l, kind in enumerate(st["layer_kind"]):
+        if kind == 1:
+            ins[l] = {"q": rng.standard_normal((n, 4, st["D"])), "k": _unit(rng.standard_normal((n, 2, st["D"]))),
+                      "v": rng.standard_normal((n, 2, st["D"]))}
+        else:
+            q, k, v, a, b, _ = _gdn_inputs(n, st["H"], st["dk"], st["dv"])
+            ins[l] = {"q": q, "k": k, "v": v, "alpha": a, "beta": b}
+    return ins
+
+
+def _cut(ins, a, b):
+    return {l: {k: x[a:b] for k, x in d.items()} for l, d in ins.items()}
+
+
+def test_zero_removal_tail_update_equals_refill():
+    """With nothing removed, causality makes the true-tail update identical to
+    a refill of the concatenated sequence (outputs, state, cache)."""
+    st = _stack()
+    N, M = 23, 9
+    ins = _tokens(N + M, st)
+    args = (st["Hkv"], st["D"], st["H"], st["dk"], st["dv"], st["R"], st["theta"])
+    _, pre = O.refill(st["layer_kind"], _cut(ins, 0, N), *args)
+    assert pre.cursor == N
+    outs, post = O.maintenance_round(pre, st["layer_kind"], [], [], _cut(ins, N, N + M), st["R"], st["theta"])
+    ref_outs, ref = O.refill(st["layer_kind"], ins, *args)
+    for l in outs:
+        np.testing.assert_allclose(outs[l], ref_outs[l][N:], atol=1e-12)
+    for l in post.states:
+        np.testing.assert_allclose(post.states[l], ref.states[l], atol=1e-12)
+    for l in post.caches:
+        np.testing.assert_allclose(post.caches[l].K, ref.caches[l].K, atol=1e-12)
+        np.testing.assert_array_equal(post.caches[l].pos, ref.caches[l].pos)
+    assert post.cursor == ref.cursor == N + M
+
+
+def test_removal_leaves_recurrent_state_and_cursor_alone():
+    """§4.1: removal does not roll back R; §4.2: holes, cursor keeps moving."""
+    st = _stack()
+    N, M = 30, 6
+    ins = _tokens(N + M, st)
+    args = (st["Hkv"], st["D"], st["H"], st["dk"], st["dv"], st["R"], st["theta"])
+    _, pre = O.refill(st["layer_kind"], _cut(ins, 0, N), *args)
+    tail = _cut(ins, N, N + M)
+    o_a, a = O.maintenance_round(pre, st["layer_kind"], [4, 12], [9, 20], tail, st["R"], st["theta"])
+    o_b, b = O.maintenance_round(pre, st["layer_kind"], [], [], tail, st["R"], st["theta"])
+    for l in a.states:
+        np.testing.assert_array_equal(a.states[l], b.states[l])
+        np.testing.assert_array_equal(o_a[l], o_b[l])
+    assert a.cursor == b.cursor == N + M
+    for l in a.caches:
+        c = a.caches[l]
+        assert c.live == N - 13 + M
+        assert list(c.pos[-M:]) == list(range(N, N + M))
+        assert np.all(np.diff(c.pos) > 0)
+        # survivors keep their stored (already rotated) keys byte for byte
+        keep = O.keep_mask(N, [4, 12], [9, 20])
+        np.testing.assert_array_equal(c.K[:, :N - 13], pre.caches[l].K[:, keep])
+    # with a removal the result is not a refill of the surviving text (§4.1)
+    surv = np.nonzero(O.keep_mask(N, [4, 12], [9, 20]))[0]
+    txt = {l: {k: np.concatenate([x[:N][surv], x[N:N + M]]) for k, x in d.items()} for l, d in ins.items()}
+    r_outs, r = O.refill(st["layer_kind"], txt, *args)
+    assert not np.allclose(r.states[0], a.states[0])
+    assert not np.allclose(r_outs[1][-M:], o_a[1])
