@@ -1,0 +1,436 @@
+#!/usr/bin/env python
+"""Throughput of true-tail memory maintenance rounds on one GB300 per rank.
+
+A step is one maintenance round (every hot-path row): removal of superseded KV
+by compaction in every attention layer, then every layer in model order
+(RoPE at the true tail + cache append + causal GQA attention for attention
+layers; chunked gated delta rule from the carried state for recurrent
+layers), then the cursor advance.  Default workload ("npc"): 4 layers in a
+3:1 delta:attention pattern (delta 16 heads, d_k = d_v = 128; attention 16
+query / 2 KV heads, head_dim 256, RoPE on 64 dims), prefix 8192 built by a
+GPU refill, 8 chained rounds each removing 1-4 spans totalling ~5% and
+appending 256 tail tokens.  Steps cycle through the chain; before round 0 of
+each chain the working state is forked from the prefix root and before every
+step L2 is flushed (a 256 MiB write), both outside the timed events.
+
+Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle
+on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from workload import synth as W  # noqa: E402
+
+METRIC = "tail tokens/sec per maintenance round and ms/round; % of HBM/tensor roofline"
+UNIT = "tail tokens/s"
+
+WORKLOAD_TEXT = {
+    "tiny": "1 delta-rule (8 heads, d 64) + 1 GQA attention layer (8/2 heads, D 64, RoPE 64), prefix 512, "
+            "2 spans totalling 64 removed, tail 64, one round",
+    "npc": "NPC context: 4 layers 3:1 (delta 16 heads d_k=d_v=128; attention 16 Q / 2 KV heads, D 256, "
+           "partial RoPE 64 dims), prefix 8192, 8 chained rounds, 1-4 spans ~5% removed, tail 256 per round",
+    "long": "long-lived character: 48 layers 3:1 (npc shapes), prefix 32768, 10 spans = 3% removed, tail 1024",
+    "pop": "population: 32 characters varlen-packed, prefixes U[2048,16384], 2-8% removed in 1-6 spans, "
+           "tails U[64,512], 12 layers 3:1 (npc shapes)",
+    "refill": "npc stack, no removals, prefix 16384 + tail 512 as a tail update",
+}
+
+
+# ----------------------------------------------------------------------------
+# accounting (algorithmic work per round)
+# ----------------------------------------------------------------------------
+def attention_flops(shape, Lp, tails):
+    """4 D Hq (M L' + M (M+1)/2) per attention layer, summed over characters."""
+    D, Hq = shape.head_dim, shape.n_q_heads
+    return sum(4.0 * D * Hq * (m * l + m * (m + 1) / 2) for l, m in zip(Lp, tails))
+
+
+def gdn_flops(shape, tails):
+    return 6.0 * shape.d_k * shape.d_v * shape.n_gdn_heads * sum(tails)
+
+
+def compaction_bytes(shape, moved_rows):
+    n_attn = len(shape.attn_layers)
+    row = shape.n_kv_heads * shape.head_dim * 2 * 2 * n_attn + 4     # K and V of every layer + position
+    return 2.0 * moved_rows * row
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def ncu_traffic(kernel_file: str, kernel: str):
+    """dram bytes per launch from a committed ncu summary, if it was taken on
+    the current source of the kernel (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)[kernel]
+        src = open(os.path.join(ROOT, "paper_2609_18935_gb300", "csrc", kernel_file), "rb").read()
+        if hashlib.sha256(src).hexdigest() != d["src_sha256"]:
+            return None
+        return d["bytes_per_launch"]
+    except Exception:
+        return None
+
+
+# ----------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.samples = []          # (t, sm, max, reasons set)
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm, mx = float(parts[1]), float(parts[2])
+            except ValueError:
+                continue
+            reasons = {n for n, v in zip(names, parts[5:9]) if v.lower().startswith("active")}
+            self.samples.append((time.time(), sm, mx, reasons))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        inside = [s for s in self.samples if t0 <= s[0] <= t1]
+        window = "timed"
+        if not inside:                      # region shorter than the sampling period
+            inside = [s for s in self.samples if t0 - 1.0 <= s[0] <= t1 + 0.25]
+            window = "timed +/- sampling period"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "window": "none"}
+        reasons = sorted(set().union(*[s[3] for s in inside]))
+        return {"sm_mhz": statistics.median(s[1] for s in inside), "sm_max_mhz": max(s[2] for s in inside),
+                "reasons": reasons, "samples": len(inside), "window": window}
+
+
+# ----------------------------------------------------------------------------
+# CPU oracle sample (cpu_baseline leg and the reference arm)
+# ----------------------------------------------------------------------------
+def oracle_sample(w, m_sample: int):
+    """Time the fp64 oracle on round 0 of character 0, restricted to the first
+    m_sample tail tokens: compaction of every attention layer + every layer.
+    Returns (seconds, tail tokens)."""
+    from oracle import kvm_oracle as O
+    s = w.shape
+    N = w.prefix_len[0]
+    caches, states = {}, {}
+    for l in s.attn_layers:
+        K, V, pos = W.prefix_cache(w, 0, l, N)
+        caches[l] = O.AttnCache(O.bf16_to_f64(K), O.bf16_to_f64(V), pos)
+    for l in s.gdn_layers:
+        states[l] = O.f32_to_f64(W.prefix_state(w, 0, l))
+    st = O.CharacterState(caches, states, N)
+    cu, sb, se, tails = W.round_plan(w, 0, [N] + [0] * (w.n_chars - 1))
+    m = min(m_sample, tails[0])
+    full = W.tail_inputs(w, 0, [m])
+    ins = {}
+    for l, kind in enumerate(s.layer_kind):
+        x = full[l]
+        ins[l] = {k: (O.bf16_to_f64(v) if v.dtype == np.uint16 else O.f32_to_f64(v)) for k, v in x.items()}
+    t0 = time.perf_counter()
+    O.maintenance_round(st, s.layer_kind, sb[cu[0]:cu[1]], se[cu[0]:cu[1]], ins, s.rotary_dim, s.rope_theta)
+    return time.perf_counter() - t0, m
+
+
+def blas_threads() -> int:
+    try:
+        from threadpoolctl import threadpool_info
+        n = [d.get("num_threads", 0) for d in threadpool_info() if d.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = W.make_workload(args.workload)
+    m = 8
+    for _ in range(args.warmup):
+        oracle_sample(w, m)
+    secs, toks = 0.0, 0
+    for _ in range(args.steps):
+        t, n = oracle_sample(w, m)
+        secs += t
+        toks += n
+    value = toks / secs
+    sample = (f"character 0, round 0 of the workload: compaction + all {len(w.shape.layer_kind)} layers for "
+              f"the first {m} tail tokens (prefix {w.prefix_len[0]}), fp64 numpy")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD_TEXT[args.workload]},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------
+# GPU arm
+# ----------------------------------------------------------------------------
+def run_kvm(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2609_18935_gb300 import build_lib, kvm
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if not os.path.exists(kvm.LIB_PATH):
+        if rank == 0:
+            build_lib.build()
+        if world > 1:
+            dist.barrier()
+    kvm.load_library()
+
+    w = W.make_workload(args.workload)
+    s = w.shape
+    plan = W.simulate_plan(w)
+    R = len(plan)
+    caps = w.capacity()
+    mk = lambda max_tail: kvm.Context(s.layer_kind, s.n_q_heads, s.n_kv_heads, s.head_dim, s.rotary_dim,
+                                      s.rope_theta, s.n_gdn_heads, s.d_k, s.d_v, caps, max_tail)
+    seed_base = 7919 * (rank + 1)        # each rank maintains its own characters
+
+    # ---- prefix root: a GPU refill of the prefix (no removals, tail = prefix)
+    N = list(w.prefix_len)
+    root = mk(sum(N))
+    ins = W.device_round_inputs(w, seed_base, N)
+    tot = sum(N)
+    outs = {l: torch.empty((tot, s.n_q_heads, s.head_dim) if k == W.ATTN else (tot, s.n_gdn_heads, s.d_v),
+                           dtype=torch.bfloat16, device="cuda") for l, k in enumerate(s.layer_kind)}
+    zero_cu = np.zeros(w.n_chars + 1, np.int32)
+    root.update_round(zero_cu, [], [], np.concatenate([[0], np.cumsum(N)]), ins, outs)
+    root.check()
+    del ins, outs
+    torch.cuda.empty_cache()
+
+    # ---- per-round inputs (device) and their pinned host copies (end to end)
+    max_tail = max(sum(p[3]) for p in plan)
+    work = mk(max_tail)
+    rounds = []
+    for r, (cu, sb, se, tails) in enumerate(plan):
+        tail_cu = np.concatenate([[0], np.cumsum(tails)]).astype(np.int32)
+        d_in = W.device_round_inputs(w, seed_base + 1 + r, tails)
+        tot = int(tail_cu[-1])
+        d_out = {l: torch.empty((tot, s.n_q_heads, s.head_dim) if k == W.ATTN else (tot, s.n_gdn_heads, s.d_v),
+                                dtype=torch.bfloat16, device="cuda") for l, k in enumerate(s.layer_kind)}
+        h_in = {l: {k: v.cpu().pin_memory() for k, v in x.items()} for l, x in d_in.items()}
+        h_out = {l: torch.empty(o.shape, dtype=o.dtype).pin_memory() for l, o in d_out.items()}
+        rounds.append(dict(cu=cu, sb=sb, se=se, tails=tails, tail_cu=tail_cu, d_in=d_in, d_out=d_out,
+                           h_in=h_in, h_out=h_out))
+    # per-round algorithmic work (live lengths follow the plan from the prefix)
+    live = list(N)
+    for rd in rounds:
+        cu, sb, se, tails = rd["cu"], rd["sb"], rd["se"], rd["tails"]
+        Lp, moved = [], 0
+        for b in range(w.n_chars):
+            rem = int((se[cu[b]:cu[b + 1]] - sb[cu[b]:cu[b + 1]]).sum())
+            Lp.append(live[b] - rem)
+            if cu[b + 1] > cu[b]:
+                moved += live[b] - rem - int(sb[cu[b]])
+            live[b] = live[b] - rem + tails[b]
+        rd["attn_flops"] = attention_flops(s, Lp, tails)        # per attention layer
+        rd["gdn_flops"] = gdn_flops(s, tails)                   # per delta-rule layer
+        rd["compact_bytes"] = compaction_bytes(s, moved)
+        rd["h2d"] = sum(t.numel() * t.element_size() for x in rd["h_in"].values() for t in x.values())
+        rd["d2h"] = sum(t.numel() * t.element_size() for t in rd["h_out"].values())
+
+    flush = torch.empty(256 << 20, dtype=torch.int8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def one_step(i, host_io):
+        r = i % R
+        rd = rounds[r]
+        if r == 0:
+            work.fork_from(root)
+        flush.fill_(i & 0x7F)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        if host_io:
+            work.update_round(rd["cu"], rd["sb"], rd["se"], rd["tail_cu"], rd["h_in"], rd["h_out"], io_on_host=True)
+        else:
+            work.update_round(rd["cu"], rd["sb"], rd["se"], rd["tail_cu"], rd["d_in"], rd["d_out"])
+        e1.record(stream)
+        return e0, e1, r
+
+    def timed(host_io):
+        for i in range(args.warmup):
+            one_step(i, host_io)
+        work.check()
+        # restart the chain so the timed steps begin at round 0
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        launches0 = work.launch_count()
+        work.profile_enable(True)
+        work.profile_read(0, reset=True)
+        t0 = time.time()
+        evs = [one_step(i, host_io) for i in range(args.steps)]
+        torch.cuda.synchronize()
+        t1 = time.time()
+        if world > 1:
+            dist.barrier()
+        work.check()
+        ms = [a.elapsed_time(b) for a, b, _ in evs]
+        kernels = {}
+        for kfam, name in enumerate(kvm.KERNEL_NAMES):
+            n, kms = work.profile_read(kfam)
+            if n:
+                kernels[name] = {"launches": n, "total_ms": kms}
+        work.profile_read(0, reset=True)
+        work.profile_enable(False)
+        launches = work.launch_count() - launches0
+        total_ms = float(sum(ms))
+        if world > 1:
+            t = torch.tensor([total_ms], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            total_ms = float(t.item())
+        return total_ms, [r for _, _, r in evs], kernels, launches, (t0, t1)
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    total_ms, rids, kernels, launches, (t0, t1) = timed(host_io=False)
+    clk = clocks.summary(t0, t1)
+    e2e_ms, e2e_rids, _, _, _ = timed(host_io=True)
+    clocks.stop()
+
+    toks_rank = sum(sum(rounds[r]["tails"]) for r in rids)
+    value = world * toks_rank / (total_ms / 1e3)
+    e2e_value = world * sum(sum(rounds[r]["tails"]) for r in e2e_rids) / (e2e_ms / 1e3)
+    hbm, tc_burst, tc_sust, peak_src = load_peaks()
+    n_attn = len(s.attn_layers)
+    attn = kernels.get("tail_attention", {"launches": 0, "total_ms": 0.0})
+    attn_flops_total = sum(rounds[r]["attn_flops"] * n_attn for r in rids)
+    achieved = attn_flops_total / (attn["total_ms"] / 1e3) / 1e12 if attn["total_ms"] > 0 else None
+    traffic = ncu_traffic("tail_attn.cu", "tail_attention")
+    roofline = {"bound": "tensor", "kernel": "tail_attention", "achieved": achieved, "peak": tc_burst,
+                "unit": "TFLOP/s", "frac": (achieved / tc_burst) if achieved else None,
+                "peak_kind": f"bf16 dense burst, {peak_src}", "traffic": traffic,
+                "algorithmic_flops_per_launch": attn_flops_total / max(1, attn["launches"])}
+    if rank != 0:
+        return
+    # ---- CPU oracle sample (rank 0 only, single GPU runs only)
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        secs, m = oracle_sample(w, 64)
+        cpu = {"value": m / secs, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+               "sample": f"character 0, round 0: compaction + all {len(s.layer_kind)} layers for the first "
+                         f"{m} of {plan[0][3][0]} tail tokens (prefix {w.prefix_len[0]}), fp64 numpy, "
+                         f"{secs:.1f} s"}
+    per_kernel = {}
+    for name, d in kernels.items():
+        per_kernel[name] = {"launches": d["launches"], "avg_us": 1e3 * d["total_ms"] / d["launches"],
+                            "share": d["total_ms"] / total_ms}
+    gdn = kernels.get("gdn_chunk_scan")
+    comp = kernels.get("kv_compact")
+    extra = {}
+    if gdn:
+        gf = sum(rounds[r]["gdn_flops"] * len(s.gdn_layers) for r in rids)
+        extra["gdn_chunk_scan_tflops"] = gf / (gdn["total_ms"] / 1e3) / 1e12
+    if comp:
+        cb = sum(rounds[r]["compact_bytes"] for r in rids)
+        extra["kv_compact_gbs"] = cb / (comp["total_ms"] / 1e3) / 1e9
+        extra["kv_compact_hbm_frac"] = extra["kv_compact_gbs"] / hbm
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD_TEXT[args.workload], "name": args.workload, "chars": w.n_chars,
+                   "layers": len(s.layer_kind), "chain_rounds": R,
+                   "l2": "flushed before every step (256 MiB write), outside the timed events",
+                   "parallelism": f"{world} independent replica(s), characters per rank fixed"},
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": UNIT,
+                "h2d_bytes_per_step": int(np.mean([rounds[r]["h2d"] for r in e2e_rids])),
+                "d2h_bytes_per_step": int(np.mean([rounds[r]["d2h"] for r in e2e_rids])),
+                "ms_per_step": e2e_ms / args.steps},
+        "gpu_launches": launches,
+        "kernels": per_kernel,
+        "derived": extra,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=64)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", choices=["kvm", "reference"], default="kvm")
+    ap.add_argument("--workload", choices=list(WORKLOAD_TEXT), default="npc")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_kvm(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,249 @@
+/*
+ * kvm.h -- C ABI of the true-tail incremental memory maintenance library.
+ *
+ * The library keeps, for a population of characters, the inference state
+ * (A_t, R_t, p_t) of a hybrid gated-delta-rule / GQA-attention model (§4.1):
+ *   A_t  live attention KV per attention layer (rotated keys and values,
+ *        bf16, plus one int32 position id per live entry, shared by all
+ *        attention layers of a character),
+ *   R_t  the recurrent state S [H][d_v][d_k] (fp32) of every delta-rule layer,
+ *   p_t  the next position id (cursor), which only moves forward (§4.2).
+ * A maintenance round removes the KV of superseded records in every attention
+ * layer (Eq. 2) and runs the M replacement tokens forward at the true tail
+ * (Eq. 3): attention layers append the tail's keys at positions p .. p+M-1
+ * and attend causally over the compacted cache plus the tail; delta-rule
+ * layers advance S from its preserved value.  Projections, norms and MLPs of
+ * the full model are outside this library: callers pass per-layer q/k/v (and
+ * the gates alpha, beta) and receive per-layer outputs.
+ *
+ * Conventions for every entry point:
+ *  - Return value: KVM_OK (0) or a KVM_E_* code.  On any error the text of
+ *    the failure is available from kvm_last_error() (thread-local), and the
+ *    context state is unchanged: all argument and span validation happens on
+ *    the host before the first launch.
+ *  - "device" pointers are CUDA global-memory addresses on the context's
+ *    device; "host" pointers are CPU memory.  bf16 tensors are passed as
+ *    void* holding IEEE bfloat16 values.  Every device pointer must be
+ *    16-byte aligned.
+ *  - stream is a cudaStream_t (NULL = legacy default stream).  Work is
+ *    enqueued asynchronously on it; the caller keeps device buffers alive
+ *    until that work completes.  A context is used from one host thread and
+ *    one stream at a time.
+ *  - Characters are packed: per-character token counts are given as
+ *    cumulative offsets cu[B+1] (cu[0] = 0), and tensors of tail tokens are
+ *    [sum M][heads][dim] with character b's tokens at rows cu[b] .. cu[b+1]-1.
+ *  - Kernels never trap.  A bounds violation or an expired bounded wait
+ *    detected on the device sets a device error word; kvm_check() reads it.
+ */
+#ifndef KVM_H
+#define KVM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int kvm_status;
+enum {
+    KVM_OK = 0,
+    KVM_E_INVAL = 1,        /* NULL or inconsistent argument, bad layer index */
+    KVM_E_SPAN = 2,         /* deletion span unsorted, overlapping, empty or outside the live cache */
+    KVM_E_CAPACITY = 3,     /* L' + M exceeds a character's capacity, or sum M exceeds max_tail_tokens */
+    KVM_E_CUDA = 4,         /* CUDA runtime / launch failure (text in kvm_last_error) */
+    KVM_E_DEVICE = 5,       /* a kernel reported a bounds violation or an expired wait */
+    KVM_E_UNSUPPORTED = 6   /* shape outside what the kernels implement */
+};
+
+enum { KVM_LAYER_GDN = 0, KVM_LAYER_ATTN = 1 };
+
+typedef struct kvm_ctx kvm_ctx;
+
+/* Model shape.  layer_kind[n_layers] lists the layers in model order.
+ * Attention layers: n_q_heads query heads share n_kv_heads KV heads (query
+ * head h reads KV head h / (n_q_heads / n_kv_heads)); head_dim D; RoPE on the
+ * first rotary_dim dims of each head, pairs (d, d + rotary_dim/2), frequency
+ * rope_theta^(-2d/rotary_dim); scores scaled by 1/sqrt(D).
+ * Delta-rule layers: n_gdn_heads heads with key dim d_k and value dim d_v.
+ * Supported: D in {64, 128, 256}; rotary_dim even, <= D; group size
+ * n_q_heads/n_kv_heads a power of two <= 64; d_k in {64, 128}; d_v a
+ * multiple of 32, <= 256. */
+typedef struct kvm_model_desc {
+    int32_t n_layers;
+    const int32_t* layer_kind;     /* host [n_layers] */
+    int32_t n_q_heads;
+    int32_t n_kv_heads;
+    int32_t head_dim;
+    int32_t rotary_dim;
+    double rope_theta;
+    int32_t n_gdn_heads;
+    int32_t d_k;
+    int32_t d_v;
+} kvm_model_desc;
+
+/* ---------------------------------------------------------------- lifetime */
+
+/* Create a context for n_chars characters on the current CUDA device.
+ * capacity: host [n_chars], KV slots per character (every attention layer);
+ * max_tail_tokens: upper bound on sum M of any later round (sizes the
+ * workspace).  The context allocates all persistent state (KV slabs,
+ * positions, S, cursors) and all workspace here, once; later calls allocate
+ * nothing.  Initial state: live length 0, cursor 0, S = 0.
+ * Errors: KVM_E_INVAL, KVM_E_UNSUPPORTED, KVM_E_CUDA (out of memory). */
+kvm_status kvm_create(const kvm_model_desc* model, int32_t n_chars,
+                      const int32_t* capacity, int32_t max_tail_tokens,
+                      kvm_ctx** out);
+
+/* Free everything the context owns.  Synchronizes the device first. */
+kvm_status kvm_destroy(kvm_ctx* ctx);
+
+/* Text of the most recent failure on this host thread ("" if none). */
+const char* kvm_last_error(void);
+
+/* ------------------------------------------------------------ state access */
+
+/* Load a character's prefix: live length `live` (<= capacity), cursor p
+ * (the next position id; must exceed every position), positions host
+ * [live] (strictly increasing, >= 0).  Keys/values are then set per layer
+ * with kvm_set_kv.  Synchronous with respect to the host arrays. */
+kvm_status kvm_load_prefix(kvm_ctx* ctx, int32_t b, int32_t live, int64_t cursor,
+                           const int32_t* positions, void* stream);
+
+/* Copy a character's live KV of attention layer `layer` (model index) in or
+ * out.  k, v: device [n_kv_heads][live][head_dim] bf16, keys in stored
+ * (already rotated) form. */
+kvm_status kvm_set_kv(kvm_ctx* ctx, int32_t layer, int32_t b, const void* k,
+                      const void* v, void* stream);
+kvm_status kvm_get_kv(kvm_ctx* ctx, int32_t layer, int32_t b, void* k_out,
+                      void* v_out, void* stream);
+
+/* Device positions of character b: pos_out device [live] int32. */
+kvm_status kvm_get_positions(kvm_ctx* ctx, int32_t b, int32_t* pos_out, void* stream);
+
+/* Recurrent state of delta-rule layer `layer` (model index), all characters:
+ * device [n_chars][n_gdn_heads][d_v][d_k] fp32. */
+kvm_status kvm_set_state(kvm_ctx* ctx, int32_t layer, const float* S, void* stream);
+kvm_status kvm_get_state(kvm_ctx* ctx, int32_t layer, float* S_out, void* stream);
+
+/* Host view of character b's live length and cursor (no synchronization). */
+kvm_status kvm_get_live(kvm_ctx* ctx, int32_t b, int32_t* live, int64_t* cursor);
+
+/* Map absolute position ranges [pos_begin, pos_end) of character b to
+ * live-index spans, checking each against the live entries (§4.2: deletion
+ * ranges are verified against live spans).  A range must cover at least one
+ * live entry and every live entry whose position lies in it; the ranges
+ * must be sorted and disjoint.  Outputs host [n].  Errors: KVM_E_SPAN. */
+kvm_status kvm_spans_from_positions(kvm_ctx* ctx, int32_t b, int32_t n,
+                                    const int64_t* pos_begin, const int64_t* pos_end,
+                                    int32_t* span_begin, int32_t* span_end);
+
+/* ------------------------------------------------------------ hot path */
+
+/* Eq. 2: remove the live entries named by the spans from every attention
+ * layer of every character, keeping survivors' bytes, positions and order
+ * (stored keys are never re-rotated, §4.2).  Survivor at old live index i
+ * moves to i - (number of removed indices < i), in place; only entries at or
+ * after a character's first removed index move.
+ * span_cu: host [n_chars+1] offsets into span_begin/span_end (host), which
+ * hold half-open live-index ranges, sorted and disjoint per character.
+ * gather_out: optional device int32 [sum L'_b], written new slot -> old slot
+ * for every surviving entry, characters packed in order; may be NULL.
+ * Errors: KVM_E_INVAL, KVM_E_SPAN (nothing launched, state unchanged). */
+kvm_status kvm_kv_compact(kvm_ctx* ctx, const int32_t* span_cu,
+                          const int32_t* span_begin, const int32_t* span_end,
+                          int32_t* gather_out, void* stream);
+
+/* Eq. 3 for one attention layer (model index `layer`): rotate the tail's
+ * queries and keys at positions p_b + i (§4.2, RoPE at the true tail),
+ * append rotated keys and values at live slots L'_b + i (L'_b = the current
+ * live length, i.e. after kv_compact) and write positions p_b + i, then
+ * o_i = sum_j softmax_j(q_i . k_j / sqrt(D)) v_j over every surviving entry
+ * and the tail's keys j <= i.
+ * tail_cu host [n_chars+1]; q device [sum M][n_q_heads][D] bf16;
+ * k_new, v_new device [sum M][n_kv_heads][D] bf16; out device
+ * [sum M][n_q_heads][D] bf16.  Does not move live lengths or cursors (see
+ * kvm_advance), so every attention layer of a round appends at the same
+ * slots.  Errors: KVM_E_INVAL, KVM_E_CAPACITY. */
+kvm_status kvm_tail_attn_prefill(kvm_ctx* ctx, int32_t layer, const int32_t* tail_cu,
+                                 const void* q, const void* k_new, const void* v_new,
+                                 void* out, void* stream);
+
+/* Eq. 3 for one gated-delta-rule layer (model index `layer`): advance each
+ * character's carried state S through its M_b tail tokens,
+ *   S_t = alpha_t S_{t-1} (I - beta_t k_t k_t^T) + beta_t v_t k_t^T,
+ *   o_t = S_t q_t,
+ * computed in chunks of 64 tokens (WY/UT form) starting at the first tail
+ * token.  S is updated in place in the context.
+ * q, k device [sum M][n_gdn_heads][d_k] bf16 (k expected unit-norm per head
+ * but not required); v device [sum M][n_gdn_heads][d_v] bf16; alpha, beta
+ * device [sum M][n_gdn_heads] fp32; out device [sum M][n_gdn_heads][d_v]
+ * bf16.  Errors: KVM_E_INVAL, KVM_E_CAPACITY. */
+kvm_status kvm_gdn_chunk_scan_from_state(kvm_ctx* ctx, int32_t layer, const int32_t* tail_cu,
+                                         const void* q, const void* k, const void* v,
+                                         const float* alpha, const float* beta,
+                                         void* out, void* stream);
+
+/* End of a round: p_b += M_b and L_b = L'_b + M_b for every character
+ * (host bookkeeping; the device positions were written by the attention
+ * layers).  tail_cu host [n_chars+1]. */
+kvm_status kvm_advance(kvm_ctx* ctx, const int32_t* tail_cu);
+
+/* One whole maintenance round: kv_compact, then every layer in model order
+ * (tail_attn_prefill or gdn_chunk_scan_from_state), then advance.
+ * Per-layer arrays are indexed by model layer; alpha/beta entries of
+ * attention layers are ignored.  io_on_host = 0: q/k/v/alpha/beta/out are
+ * device pointers.  io_on_host = 1: they are host pointers (pinned memory
+ * for asynchronous copies); the library copies each layer's inputs into its
+ * own device staging buffers and the layer's output back, on `stream`. */
+typedef struct kvm_round {
+    const int32_t* span_cu;        /* host [n_chars+1] */
+    const int32_t* span_begin;     /* host */
+    const int32_t* span_end;       /* host */
+    const int32_t* tail_cu;        /* host [n_chars+1] */
+    const void* const* q;          /* [n_layers] */
+    const void* const* k;          /* [n_layers] */
+    const void* const* v;          /* [n_layers] */
+    const float* const* alpha;     /* [n_layers] */
+    const float* const* beta;      /* [n_layers] */
+    void* const* out;              /* [n_layers] */
+    int32_t io_on_host;
+    int32_t* gather_out;           /* optional device, see kvm_kv_compact */
+} kvm_round;
+
+kvm_status kvm_update_round(kvm_ctx* ctx, const kvm_round* round, void* stream);
+
+/* Copy the whole state of `src` into `dst`: every character's live KV,
+ * positions, recurrent states, live lengths and cursors (§4.2: task-specific
+ * continuations branch from a maintained root).  Both contexts must have the
+ * same model shape, character count and capacities (max_tail_tokens may
+ * differ).  Enqueued on `stream`; dst's previous state is overwritten.
+ * Errors: KVM_E_INVAL (shapes differ). */
+kvm_status kvm_fork(kvm_ctx* dst, const kvm_ctx* src, void* stream);
+
+/* Per-kernel timing for diagnostics.  While enabled, each kernel launch of
+ * the library is bracketed by a pair of CUDA events on its stream.
+ * kvm_profile_read synchronizes the device and returns, for one kernel
+ * family (KVM_K_*), the number of launches and their summed device time in
+ * milliseconds since the last reset; reset != 0 clears every family.
+ * Events come from a pool made at enable time (4096 launches between
+ * reads); launches beyond it are counted but not timed. */
+enum { KVM_K_COMPACT = 0, KVM_K_ROPE_APPEND = 1, KVM_K_ATTENTION = 2, KVM_K_ATTN_COMBINE = 3,
+       KVM_K_GDN = 4, KVM_K_GATHER = 5, KVM_K_COUNT = 6 };
+kvm_status kvm_profile_enable(kvm_ctx* ctx, int32_t enable);
+kvm_status kvm_profile_read(kvm_ctx* ctx, int32_t kernel, int64_t* launches, double* total_ms,
+                            int32_t reset);
+
+/* Synchronize `stream` and read the device error word; returns KVM_E_DEVICE
+ * (and clears the word) if a kernel reported a violation since the last
+ * check. */
+kvm_status kvm_check(kvm_ctx* ctx, void* stream);
+
+/* Number of kernel launches the library has enqueued since creation
+ * (diagnostics for the benchmark). */
+int64_t kvm_launch_count(const kvm_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVM_H */

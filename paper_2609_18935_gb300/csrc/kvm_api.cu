@@ -1,0 +1,817 @@
+// Host runtime and C ABI of the maintenance library (include/kvm.h).
+//
+// The context owns a character population's state (A_t, R_t, p_t) (§4.1):
+//   K, V    [n_attn][Hkv][T_cap][D] bf16   (character b at slot offset cap_off[b])
+//   pos     [T_cap] int32                  (shared by every attention layer)
+//   S       [n_gdn][B][H][d_v][d_k] fp32
+//   cursor, live length and a host mirror of positions per character.
+// Every argument and span is validated here before anything is enqueued, so a
+// rejected call leaves the state untouched.  Per-round descriptors travel to
+// the kernels as kernel parameters: nothing is allocated or uploaded per call.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/kvm.h"
+#include "kvm_internal.cuh"
+
+using namespace kvm;
+
+namespace {
+
+thread_local std::string g_err;
+
+kvm_status fail(kvm_status code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return code;
+}
+
+#define CUDA_TRY(expr)                                                                  \
+    do {                                                                                \
+        cudaError_t e_ = (expr);                                                        \
+        if (e_ != cudaSuccess)                                                          \
+            return fail(KVM_E_CUDA, "%s failed: %s", #expr, cudaGetErrorString(e_));     \
+    } while (0)
+
+#define LAUNCH_CHECK(ctx)                                                                \
+    do {                                                                                 \
+        cudaError_t e_ = cudaGetLastError();                                             \
+        if (e_ != cudaSuccess) return fail(KVM_E_CUDA, "kernel launch failed: %s", cudaGetErrorString(e_)); \
+    } while (0)
+
+constexpr int kItemCap = 1216;      // work items that keep a partial accumulator (8 per SM at 152 SMs)
+
+}  // namespace
+
+struct kvm_ctx {
+    int device = 0;
+    int num_sms = 0;
+    // model
+    int n_layers = 0;
+    std::vector<int> kind, attn_idx, gdn_idx;
+    int n_attn = 0, n_gdn = 0;
+    int Hq = 0, Hkv = 0, D = 0, R = 0, g = 0;
+    double theta = 0;
+    int H = 0, dk = 0, dv = 0;
+    // population
+    int B = 0;
+    std::vector<int> cap, cap_off;
+    int64_t T_cap = 0;
+    int max_tail = 0;
+    std::vector<int> live;
+    std::vector<int64_t> cursor;
+    std::vector<std::vector<int32_t>> hpos;
+    // device state
+    __nv_bfloat16* K = nullptr;
+    __nv_bfloat16* V = nullptr;
+    int32_t* pos = nullptr;
+    float* S = nullptr;
+    // workspace
+    __nv_bfloat16* q_rot = nullptr;
+    float* part_o = nullptr;
+    float* part_ml = nullptr;
+    int32_t* tickets = nullptr;
+    uint32_t* flags = nullptr;
+    std::vector<int> flag_off;
+    uint32_t epoch = 0;
+    int32_t* err = nullptr;
+    // staging for host-resident round inputs
+    void* stage_in[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
+    void* stage_out = nullptr;
+    size_t stage_bytes[5] = {0, 0, 0, 0, 0};
+    size_t stage_out_bytes = 0;
+    double inv_freq[kMaxRotaryHalf] = {};
+    int64_t launches = 0;
+    int rows_kv = 0, rows_pos = 0;
+    // per-kernel timing (kvm_profile_*)
+    bool prof = false;
+    std::vector<cudaEvent_t> ev;          // 2 per timed launch
+    std::vector<int> ev_kind;             // kind of each recorded pair
+    int64_t prof_launches[KVM_K_COUNT] = {};
+};
+
+namespace {
+
+template <typename T>
+cudaError_t alloc_zero(T** p, size_t count) {
+    if (count == 0) { *p = nullptr; return cudaSuccess; }
+    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T));
+    if (e != cudaSuccess) return e;
+    return cudaMemset(*p, 0, count * sizeof(T));
+}
+
+void free_all(kvm_ctx* c) {
+    void* ptrs[] = {c->K, c->V, c->pos, c->S, c->q_rot, c->part_o, c->part_ml, c->tickets,
+                    c->flags, c->err, c->stage_in[0], c->stage_in[1], c->stage_in[2],
+                    c->stage_in[3], c->stage_in[4], c->stage_out};
+    for (void* p : ptrs)
+        if (p) cudaFree(p);
+    for (cudaEvent_t e : c->ev) cudaEventDestroy(e);
+    c->ev.clear();
+}
+
+kvm_status check_tail_cu(const kvm_ctx* c, const int32_t* tail_cu, int* total) {
+    if (!tail_cu) return fail(KVM_E_INVAL, "tail_cu is NULL");
+    if (tail_cu[0] != 0) return fail(KVM_E_INVAL, "tail_cu[0] must be 0");
+    for (int b = 0; b < c->B; ++b) {
+        const int m = tail_cu[b + 1] - tail_cu[b];
+        if (m < 0) return fail(KVM_E_INVAL, "tail_cu not monotone at character %d", b);
+    }
+    *total = tail_cu[c->B];
+    if (*total > c->max_tail)
+        return fail(KVM_E_CAPACITY, "sum M = %d exceeds max_tail_tokens = %d", *total, c->max_tail);
+    return KVM_OK;
+}
+
+kvm_status check_layer(const kvm_ctx* c, int layer, int want) {
+    if (layer < 0 || layer >= c->n_layers) return fail(KVM_E_INVAL, "layer %d out of range", layer);
+    if (c->kind[layer] != want)
+        return fail(KVM_E_INVAL, "layer %d is not a %s layer", layer,
+                    want == KVM_LAYER_ATTN ? "attention" : "delta-rule");
+    return KVM_OK;
+}
+
+constexpr int kProfPool = 4096;
+
+// Bracket one launch with a pair of events when profiling is on.
+int prof_begin(kvm_ctx* c, int kind, cudaStream_t s) {
+    ++c->launches;
+    if (!c->prof) return -1;
+    ++c->prof_launches[kind];
+    const int slot = (int)c->ev_kind.size();
+    if (slot >= kProfPool) return -1;
+    c->ev_kind.push_back(kind);
+    cudaEventRecord(c->ev[2 * slot], s);
+    return slot;
+}
+
+void prof_end(kvm_ctx* c, int slot, cudaStream_t s) {
+    if (slot >= 0) cudaEventRecord(c->ev[2 * slot + 1], s);
+}
+
+// Validate one round's spans and build the per-character segment tables.
+struct SpanPlan {
+    std::vector<int> L_new, first, seg_off, n_seg;
+    std::vector<int32_t> seg_start, seg_shift;
+};
+
+kvm_status plan_spans(const kvm_ctx* c, const int32_t* span_cu, const int32_t* sb, const int32_t* se,
+                      SpanPlan& pl) {
+    if (!span_cu) return fail(KVM_E_INVAL, "span_cu is NULL");
+    if (span_cu[0] != 0) return fail(KVM_E_INVAL, "span_cu[0] must be 0");
+    const int total = span_cu[c->B];
+    if (total < 0) return fail(KVM_E_INVAL, "negative span count");
+    if (total > kMaxSpans) return fail(KVM_E_INVAL, "%d spans exceed the per-round limit %d", total, kMaxSpans);
+    if (total > 0 && (!sb || !se)) return fail(KVM_E_INVAL, "span arrays are NULL");
+    pl.L_new.assign(c->B, 0);
+    pl.first.assign(c->B, 0);
+    pl.seg_off.assign(c->B, 0);
+    pl.n_seg.assign(c->B, 0);
+    pl.seg_start.clear();
+    pl.seg_shift.clear();
+    for (int b = 0; b < c->B; ++b) {
+        const int s0 = span_cu[b], s1 = span_cu[b + 1];
+        if (s1 < s0) return fail(KVM_E_INVAL, "span_cu not monotone at character %d", b);
+        const int L = c->live[b];
+        int removed = 0, prev_end = 0;
+        pl.seg_off[b] = (int)pl.seg_start.size();
+        pl.n_seg[b] = s1 - s0;
+        for (int k = s0; k < s1; ++k) {
+            const int lo = sb[k], hi = se[k];
+            if (!(0 <= lo && lo < hi && hi <= L))
+                return fail(KVM_E_SPAN, "character %d span %d [%d,%d) empty or outside live [0,%d)", b, k - s0,
+                            lo, hi, L);
+            if (k > s0 && lo < prev_end)
+                return fail(KVM_E_SPAN, "character %d span %d overlaps or precedes the previous span", b, k - s0);
+            prev_end = hi;
+            removed += hi - lo;
+            // survivors after this span: new index (hi - removed) onward come from + removed
+            pl.seg_start.push_back(hi - removed);
+            pl.seg_shift.push_back(removed);
+        }
+        pl.L_new[b] = L - removed;
+        pl.first[b] = (s1 > s0) ? sb[s0] : pl.L_new[b];
+    }
+    return KVM_OK;
+}
+
+}  // namespace
+
+// ============================================================================
+// lifetime
+// ============================================================================
+extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const int32_t* capacity,
+                                 int32_t max_tail_tokens, kvm_ctx** out) {
+    if (!m || !capacity || !out) return fail(KVM_E_INVAL, "NULL argument");
+    *out = nullptr;
+    if (m->n_layers <= 0 || !m->layer_kind) return fail(KVM_E_INVAL, "model has no layers");
+    if (n_chars <= 0 || n_chars > kMaxChars) return fail(KVM_E_INVAL, "n_chars must be in [1,%d]", kMaxChars);
+    if (max_tail_tokens <= 0) return fail(KVM_E_INVAL, "max_tail_tokens must be positive");
+    kvm_ctx* c = new kvm_ctx();
+    c->n_layers = m->n_layers;
+    for (int l = 0; l < m->n_layers; ++l) {
+        const int k = m->layer_kind[l];
+        if (k != KVM_LAYER_ATTN && k != KVM_LAYER_GDN) { delete c; return fail(KVM_E_INVAL, "bad layer kind"); }
+        c->kind.push_back(k);
+        c->attn_idx.push_back(k == KVM_LAYER_ATTN ? c->n_attn++ : -1);
+        c->gdn_idx.push_back(k == KVM_LAYER_GDN ? c->n_gdn++ : -1);
+    }
+    if (c->n_attn > 0) {
+        c->Hq = m->n_q_heads; c->Hkv = m->n_kv_heads; c->D = m->head_dim; c->R = m->rotary_dim;
+        c->theta = m->rope_theta;
+        if (c->Hkv <= 0 || c->Hq <= 0 || c->Hq % c->Hkv) { delete c; return fail(KVM_E_UNSUPPORTED, "n_q_heads must be a multiple of n_kv_heads"); }
+        c->g = c->Hq / c->Hkv;
+        if (c->g > 64 || (c->g & (c->g - 1))) { delete c; return fail(KVM_E_UNSUPPORTED, "group size must be a power of two <= 64"); }
+        if (c->D != 64 && c->D != 128 && c->D != 256) { delete c; return fail(KVM_E_UNSUPPORTED, "head_dim must be 64, 128 or 256"); }
+        if (c->R < 0 || c->R > c->D || (c->R & 1)) { delete c; return fail(KVM_E_UNSUPPORTED, "rotary_dim must be even and <= head_dim"); }
+        if (!(c->theta > 0)) { delete c; return fail(KVM_E_INVAL, "rope_theta must be positive"); }
+        for (int d = 0; d < c->R / 2; ++d) c->inv_freq[d] = std::pow(c->theta, -2.0 * d / c->R);
+    }
+    if (c->n_gdn > 0) {
+        c->H = m->n_gdn_heads; c->dk = m->d_k; c->dv = m->d_v;
+        if (c->H <= 0) { delete c; return fail(KVM_E_INVAL, "n_gdn_heads must be positive"); }
+        if (c->dk != 64 && c->dk != 128) { delete c; return fail(KVM_E_UNSUPPORTED, "d_k must be 64 or 128"); }
+        if (c->dv <= 0 || c->dv % 32 || c->dv > 256) { delete c; return fail(KVM_E_UNSUPPORTED, "d_v must be a multiple of 32, <= 256"); }
+    }
+    c->B = n_chars;
+    c->max_tail = max_tail_tokens;
+    for (int b = 0; b < n_chars; ++b) {
+        if (capacity[b] <= 0) { delete c; return fail(KVM_E_INVAL, "capacity of character %d must be positive", b); }
+        const int cp = (capacity[b] + 63) / 64 * 64;   // slab offsets stay 64-row aligned
+        c->cap.push_back(cp);
+        c->cap_off.push_back((int)c->T_cap);
+        c->T_cap += cp;
+    }
+    if (c->T_cap > INT32_MAX) { delete c; return fail(KVM_E_CAPACITY, "total capacity too large"); }
+    c->live.assign(n_chars, 0);
+    c->cursor.assign(n_chars, 0);
+    c->hpos.assign(n_chars, {});
+
+    cudaError_t e = cudaGetDevice(&c->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess) { delete c; return fail(KVM_E_CUDA, "no CUDA device: %s", cudaGetErrorString(e)); }
+
+    const size_t kv_elems = (size_t)c->n_attn * c->Hkv * c->T_cap * c->D;
+    const int vec_per_row = c->D * 2 / 16;
+    c->rows_kv = c->n_attn ? kCompactVecPerChunk / std::max(vec_per_row, 1) : 1;
+    c->rows_pos = kCompactVecPerChunk;
+    const int n_kv_slabs = 2 * c->n_attn * c->Hkv;
+    size_t n_flags = 0;
+    for (int b = 0; b < n_chars; ++b) {
+        c->flag_off.push_back((int)n_flags);
+        n_flags += (size_t)n_kv_slabs * ((c->cap[b] + c->rows_kv - 1) / c->rows_kv) +
+                   (c->cap[b] + c->rows_pos - 1) / c->rows_pos;
+    }
+    const size_t attn_in = (size_t)max_tail_tokens * std::max(c->Hq * c->D, c->H * c->dk);
+    const size_t kv_in = (size_t)max_tail_tokens * std::max(c->Hkv * c->D, c->H * c->dk);
+    const size_t v_in = (size_t)max_tail_tokens * std::max(c->Hkv * c->D, c->H * c->dv);
+    const size_t out_n = (size_t)max_tail_tokens * std::max(c->Hq * c->D, c->H * c->dv);
+    e = cudaSuccess;
+    if (e == cudaSuccess) e = alloc_zero(&c->K, kv_elems);
+    if (e == cudaSuccess) e = alloc_zero(&c->V, kv_elems);
+    if (e == cudaSuccess) e = alloc_zero(&c->pos, c->n_attn ? (size_t)c->T_cap : 0);
+    if (e == cudaSuccess) e = alloc_zero(&c->S, (size_t)c->n_gdn * n_chars * c->H * c->dv * c->dk);
+    if (e == cudaSuccess) e = alloc_zero(&c->q_rot, c->n_attn ? (size_t)max_tail_tokens * c->Hq * c->D : 0);
+    if (e == cudaSuccess) e = alloc_zero(&c->part_o, c->n_attn ? (size_t)kItemCap * 64 * c->D : 0);
+    if (e == cudaSuccess) e = alloc_zero(&c->part_ml, c->n_attn ? (size_t)kItemCap * 64 * 2 : 0);
+    if (e == cudaSuccess) e = alloc_zero(&c->tickets, (size_t)n_chars * (n_kv_slabs + 1));
+    if (e == cudaSuccess) e = alloc_zero(&c->flags, n_flags);
+    if (e == cudaSuccess) e = alloc_zero(&c->err, 1);
+    c->stage_bytes[0] = attn_in * 2;   // q
+    c->stage_bytes[1] = kv_in * 2;     // k
+    c->stage_bytes[2] = v_in * 2;      // v
+    c->stage_bytes[3] = (size_t)max_tail_tokens * std::max(c->H, 1) * 4;   // alpha
+    c->stage_bytes[4] = c->stage_bytes[3];                                  // beta
+    c->stage_out_bytes = out_n * 2;
+    for (int i = 0; i < 5 && e == cudaSuccess; ++i)
+        e = cudaMalloc(&c->stage_in[i], c->stage_bytes[i]);
+    if (e == cudaSuccess) e = cudaMalloc(&c->stage_out, c->stage_out_bytes);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        free_all(c);
+        delete c;
+        return fail(KVM_E_CUDA, "allocation failed: %s", cudaGetErrorString(e));
+    }
+    *out = c;
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_destroy(kvm_ctx* c) {
+    if (!c) return KVM_OK;
+    cudaDeviceSynchronize();
+    free_all(c);
+    delete c;
+    return KVM_OK;
+}
+
+extern "C" const char* kvm_last_error(void) { return g_err.c_str(); }
+
+extern "C" int64_t kvm_launch_count(const kvm_ctx* c) { return c ? c->launches : 0; }
+
+// ============================================================================
+// state access
+// ============================================================================
+extern "C" kvm_status kvm_load_prefix(kvm_ctx* c, int32_t b, int32_t live, int64_t cursor,
+                                      const int32_t* positions, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    if (live < 0 || live > c->cap[b]) return fail(KVM_E_CAPACITY, "live %d exceeds capacity %d", live, c->cap[b]);
+    if (live > 0 && !positions) return fail(KVM_E_INVAL, "positions is NULL");
+    for (int i = 0; i < live; ++i) {
+        if (positions[i] < 0 || (i > 0 && positions[i] <= positions[i - 1]))
+            return fail(KVM_E_INVAL, "positions must be non-negative and strictly increasing");
+    }
+    if (live > 0 && cursor <= positions[live - 1]) return fail(KVM_E_INVAL, "cursor must exceed every position");
+    if (cursor < 0 || cursor + c->max_tail > INT32_MAX) return fail(KVM_E_INVAL, "cursor out of range");
+    cudaStream_t s = (cudaStream_t)stream;
+    if (c->n_attn && live > 0) {
+        CUDA_TRY(cudaMemcpyAsync(c->pos + c->cap_off[b], positions, (size_t)live * 4, cudaMemcpyHostToDevice, s));
+        CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    c->live[b] = live;
+    c->cursor[b] = cursor;
+    c->hpos[b].assign(positions, positions + live);
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_set_kv(kvm_ctx* c, int32_t layer, int32_t b, const void* k, const void* v,
+                                 void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    kvm_status st = check_layer(c, layer, KVM_LAYER_ATTN);
+    if (st) return st;
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    const int L = c->live[b];
+    if (L == 0) return KVM_OK;
+    if (!k || !v) return fail(KVM_E_INVAL, "NULL k or v");
+    const size_t row = (size_t)c->D * 2;
+    const size_t slab = (size_t)c->T_cap * row;
+    const int a = c->attn_idx[layer];
+    char* kd = reinterpret_cast<char*>(c->K) + ((size_t)a * c->Hkv) * slab + (size_t)c->cap_off[b] * row;
+    char* vd = reinterpret_cast<char*>(c->V) + ((size_t)a * c->Hkv) * slab + (size_t)c->cap_off[b] * row;
+    cudaStream_t s = (cudaStream_t)stream;
+    CUDA_TRY(cudaMemcpy2DAsync(kd, slab, k, L * row, L * row, c->Hkv, cudaMemcpyDeviceToDevice, s));
+    CUDA_TRY(cudaMemcpy2DAsync(vd, slab, v, L * row, L * row, c->Hkv, cudaMemcpyDeviceToDevice, s));
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_get_kv(kvm_ctx* c, int32_t layer, int32_t b, void* k, void* v, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    kvm_status st = check_layer(c, layer, KVM_LAYER_ATTN);
+    if (st) return st;
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    const int L = c->live[b];
+    if (L == 0) return KVM_OK;
+    if (!k || !v) return fail(KVM_E_INVAL, "NULL k or v");
+    const size_t row = (size_t)c->D * 2;
+    const size_t slab = (size_t)c->T_cap * row;
+    const int a = c->attn_idx[layer];
+    const char* ks = reinterpret_cast<const char*>(c->K) + ((size_t)a * c->Hkv) * slab + (size_t)c->cap_off[b] * row;
+    const char* vs = reinterpret_cast<const char*>(c->V) + ((size_t)a * c->Hkv) * slab + (size_t)c->cap_off[b] * row;
+    cudaStream_t s = (cudaStream_t)stream;
+    CUDA_TRY(cudaMemcpy2DAsync(k, L * row, ks, slab, L * row, c->Hkv, cudaMemcpyDeviceToDevice, s));
+    CUDA_TRY(cudaMemcpy2DAsync(v, L * row, vs, slab, L * row, c->Hkv, cudaMemcpyDeviceToDevice, s));
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_get_positions(kvm_ctx* c, int32_t b, int32_t* out, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    if (c->live[b] == 0 || c->n_attn == 0) return KVM_OK;
+    if (!out) return fail(KVM_E_INVAL, "NULL output");
+    CUDA_TRY(cudaMemcpyAsync(out, c->pos + c->cap_off[b], (size_t)c->live[b] * 4, cudaMemcpyDeviceToDevice,
+                             (cudaStream_t)stream));
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_set_state(kvm_ctx* c, int32_t layer, const float* S, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    kvm_status st = check_layer(c, layer, KVM_LAYER_GDN);
+    if (st) return st;
+    if (!S) return fail(KVM_E_INVAL, "NULL state");
+    const size_t n = (size_t)c->B * c->H * c->dv * c->dk;
+    CUDA_TRY(cudaMemcpyAsync(c->S + (size_t)c->gdn_idx[layer] * n, S, n * 4, cudaMemcpyDeviceToDevice,
+                             (cudaStream_t)stream));
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_get_state(kvm_ctx* c, int32_t layer, float* S, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    kvm_status st = check_layer(c, layer, KVM_LAYER_GDN);
+    if (st) return st;
+    if (!S) return fail(KVM_E_INVAL, "NULL state");
+    const size_t n = (size_t)c->B * c->H * c->dv * c->dk;
+    CUDA_TRY(cudaMemcpyAsync(S, c->S + (size_t)c->gdn_idx[layer] * n, n * 4, cudaMemcpyDeviceToDevice,
+                             (cudaStream_t)stream));
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_get_live(kvm_ctx* c, int32_t b, int32_t* live, int64_t* cursor) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    if (live) *live = c->live[b];
+    if (cursor) *cursor = c->cursor[b];
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_spans_from_positions(kvm_ctx* c, int32_t b, int32_t n, const int64_t* pb,
+                                               const int64_t* pe, int32_t* sb, int32_t* se) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    if (n < 0) return fail(KVM_E_INVAL, "negative count");
+    if (n > 0 && (!pb || !pe || !sb || !se)) return fail(KVM_E_INVAL, "NULL argument");
+    const std::vector<int32_t>& P = c->hpos[b];
+    int64_t prev_end = INT64_MIN;
+    for (int i = 0; i < n; ++i) {
+        if (pb[i] >= pe[i]) return fail(KVM_E_SPAN, "position range %d is empty", i);
+        if (pb[i] < prev_end) return fail(KVM_E_SPAN, "position range %d overlaps or precedes the previous one", i);
+        prev_end = pe[i];
+        const int lo = (int)(std::lower_bound(P.begin(), P.end(), pb[i]) - P.begin());
+        const int hi = (int)(std::lower_bound(P.begin(), P.end(), pe[i]) - P.begin());
+        if (hi <= lo) return fail(KVM_E_SPAN, "position range %d covers no live entry", i);
+        sb[i] = lo;
+        se[i] = hi;
+    }
+    return KVM_OK;
+}
+
+// ============================================================================
+// hot path
+// ============================================================================
+namespace {
+
+kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, const int32_t* send,
+                      int32_t* gather_out, cudaStream_t s) {
+    SpanPlan pl;
+    kvm_status st = plan_spans(c, span_cu, sbeg, send, pl);
+    if (st) return st;
+
+    if (c->n_attn > 0) {
+        thread_local static CompactParams p;   // large parameter block, copied into the launch
+        std::memset(&p, 0, sizeof p);
+        p.n_chars = c->B;
+        p.n_kv_slabs = 2 * c->n_attn * c->Hkv;
+        p.vec_per_row = c->D * 2 / 16;
+        p.rows_kv = c->rows_kv;
+        p.rows_pos = c->rows_pos;
+        p.epoch = ++c->epoch;
+        p.slab_rows = c->T_cap;
+        p.K = reinterpret_cast<uint4*>(c->K);
+        p.V = reinterpret_cast<uint4*>(c->V);
+        p.pos = c->pos;
+        p.tickets = c->tickets;
+        p.flags = c->flags;
+        p.err = c->err;
+        int blk = 0;
+        for (int b = 0; b < c->B; ++b) {
+            CompactChar& ch = p.ch[b];
+            const int moved = pl.n_seg[b] > 0 ? pl.L_new[b] - pl.first[b] : 0;
+            ch.L_new = pl.L_new[b];
+            ch.first = pl.first[b];
+            ch.seg_off = pl.seg_off[b];
+            ch.n_seg = pl.n_seg[b];
+            ch.cap_off = c->cap_off[b];
+            ch.chunks_kv = (moved + p.rows_kv - 1) / p.rows_kv;
+            ch.chunks_pos = (moved + p.rows_pos - 1) / p.rows_pos;
+            ch.blk_off = blk;
+            ch.flag_off = c->flag_off[b];
+            blk += p.n_kv_slabs * ch.chunks_kv + ch.chunks_pos;
+        }
+        p.total_blocks = blk;
+        std::copy(pl.seg_start.begin(), pl.seg_start.end(), p.seg_start);
+        std::copy(pl.seg_shift.begin(), pl.seg_shift.end(), p.seg_shift);
+        if (blk > 0) {
+            const int ps = prof_begin(c, KVM_K_COMPACT, s);
+            launch_kv_compact(p, s);
+            prof_end(c, ps, s);
+            LAUNCH_CHECK(c);
+        }
+    }
+    if (gather_out) {
+        thread_local static GatherParams gp;
+        std::memset(&gp, 0, sizeof gp);
+        gp.n_chars = c->B;
+        int tot = 0;
+        for (int b = 0; b < c->B; ++b) {
+            gp.out_off[b] = tot;
+            gp.first[b] = pl.first[b];
+            gp.seg_off[b] = pl.seg_off[b];
+            gp.n_seg[b] = pl.n_seg[b];
+            tot += pl.L_new[b];
+        }
+        gp.out_off[c->B] = tot;
+        gp.total = tot;
+        gp.out = gather_out;
+        std::copy(pl.seg_start.begin(), pl.seg_start.end(), gp.seg_start);
+        std::copy(pl.seg_shift.begin(), pl.seg_shift.end(), gp.seg_shift);
+        if (tot > 0) {
+            const int ps = prof_begin(c, KVM_K_GATHER, s);
+            launch_gather_map(gp, s);
+            prof_end(c, ps, s);
+            LAUNCH_CHECK(c);
+        }
+    }
+    // host bookkeeping: live lengths and the position mirror
+    for (int b = 0; b < c->B; ++b) {
+        if (pl.n_seg[b] == 0) continue;
+        std::vector<int32_t>& P = c->hpos[b];
+        std::vector<int32_t> keep;
+        keep.reserve(pl.L_new[b]);
+        int k = span_cu[b];
+        for (int i = 0; i < (int)P.size(); ++i) {
+            while (k < span_cu[b + 1] && i >= send[k]) ++k;
+            if (k < span_cu[b + 1] && i >= sbeg[k]) continue;
+            keep.push_back(P[i]);
+        }
+        P.swap(keep);
+        c->live[b] = pl.L_new[b];
+    }
+    return KVM_OK;
+}
+
+kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, const void* k_new,
+                        const void* v_new, void* out, cudaStream_t s) {
+    kvm_status st = check_layer(c, layer, KVM_LAYER_ATTN);
+    if (st) return st;
+    int total = 0;
+    st = check_tail_cu(c, tail_cu, &total);
+    if (st) return st;
+    for (int b = 0; b < c->B; ++b) {
+        const int m = tail_cu[b + 1] - tail_cu[b];
+        if (c->live[b] + m > c->cap[b])
+            return fail(KVM_E_CAPACITY, "character %d: live %d + tail %d exceeds capacity %d", b, c->live[b], m,
+                        c->cap[b]);
+        if (c->cursor[b] + m > INT32_MAX) return fail(KVM_E_CAPACITY, "character %d: position ids overflow", b);
+    }
+    if (total == 0) return KVM_OK;
+    if (!q || !k_new || !v_new || !out) return fail(KVM_E_INVAL, "NULL tensor");
+
+    thread_local static AttnParams p;
+    std::memset(&p, 0, sizeof p);
+    const int a = c->attn_idx[layer];
+    p.n_chars = c->B;
+    p.Hq = c->Hq; p.Hkv = c->Hkv; p.D = c->D; p.R = c->R; p.g = c->g;
+    p.tok_per_tile = 64 / c->g;
+    p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->D));
+    p.slab_rows = c->T_cap;
+    p.q = static_cast<const __nv_bfloat16*>(q);
+    p.k_new = static_cast<const __nv_bfloat16*>(k_new);
+    p.v_new = static_cast<const __nv_bfloat16*>(v_new);
+    p.q_rot = c->q_rot;
+    p.K = c->K + (size_t)a * c->Hkv * c->T_cap * c->D;
+    p.V = c->V + (size_t)a * c->Hkv * c->T_cap * c->D;
+    p.pos = c->pos;
+    p.out = static_cast<__nv_bfloat16*>(out);
+    p.part_o = c->part_o;
+    p.part_ml = c->part_ml;
+    p.err = c->err;
+    for (int d = 0; d < c->R / 2; ++d) p.inv_freq[d] = c->inv_freq[d];
+    int tiles = 0;
+    for (int b = 0; b < c->B; ++b) {
+        AttnChar& ch = p.ch[b];
+        ch.L_prev = c->live[b];
+        ch.M = tail_cu[b + 1] - tail_cu[b];
+        ch.tail_off = tail_cu[b];
+        ch.cap_off = c->cap_off[b];
+        ch.p = c->cursor[b];
+        ch.n_qtiles = (ch.M + p.tok_per_tile - 1) / p.tok_per_tile;
+        tiles += c->Hkv * ch.n_qtiles;
+    }
+    // key splits: fill about two waves of blocks when the tiles alone do not
+    int split = 1;
+    if (tiles < 2 * c->num_sms) split = std::min(16, (2 * c->num_sms + tiles - 1) / tiles);
+    while (split > 1 && (size_t)tiles * split > (size_t)kItemCap) --split;
+    p.n_split = split;
+    int items = 0;
+    for (int b = 0; b < c->B; ++b) {
+        p.ch[b].item_off = items;
+        items += c->Hkv * p.ch[b].n_qtiles * split;
+    }
+    p.n_items = items;
+
+    int ps = prof_begin(c, KVM_K_ROPE_APPEND, s);
+    launch_rope_append(p, total, s);
+    prof_end(c, ps, s);
+    LAUNCH_CHECK(c);
+    ps = prof_begin(c, KVM_K_ATTENTION, s);
+    launch_tail_attention(p, s);
+    prof_end(c, ps, s);
+    LAUNCH_CHECK(c);
+    if (split > 1) {
+        ps = prof_begin(c, KVM_K_ATTN_COMBINE, s);
+        launch_attn_combine(p, tiles, s);
+        prof_end(c, ps, s);
+        LAUNCH_CHECK(c);
+    }
+    return KVM_OK;
+}
+
+kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, const void* k, const void* v,
+                  const float* alpha, const float* beta, void* out, cudaStream_t s) {
+    kvm_status st = check_layer(c, layer, KVM_LAYER_GDN);
+    if (st) return st;
+    int total = 0;
+    st = check_tail_cu(c, tail_cu, &total);
+    if (st) return st;
+    if (total == 0) return KVM_OK;
+    if (!q || !k || !v || !alpha || !beta || !out) return fail(KVM_E_INVAL, "NULL tensor");
+    thread_local static GdnParams p;
+    std::memset(&p, 0, sizeof p);
+    p.n_chars = c->B;
+    p.H = c->H; p.dk = c->dk; p.dv = c->dv;
+    p.q = static_cast<const __nv_bfloat16*>(q);
+    p.k = static_cast<const __nv_bfloat16*>(k);
+    p.v = static_cast<const __nv_bfloat16*>(v);
+    p.alpha = alpha;
+    p.beta = beta;
+    p.out = static_cast<__nv_bfloat16*>(out);
+    p.S = c->S + (size_t)c->gdn_idx[layer] * c->B * c->H * c->dv * c->dk;
+    p.err = c->err;
+    for (int b = 0; b < c->B; ++b) {
+        p.ch[b].M = tail_cu[b + 1] - tail_cu[b];
+        p.ch[b].tail_off = tail_cu[b];
+    }
+    const int ps = prof_begin(c, KVM_K_GDN, s);
+    launch_gdn_chunk_scan(p, s);
+    prof_end(c, ps, s);
+    LAUNCH_CHECK(c);
+    return KVM_OK;
+}
+
+void do_advance(kvm_ctx* c, const int32_t* tail_cu) {
+    for (int b = 0; b < c->B; ++b) {
+        const int m = tail_cu[b + 1] - tail_cu[b];
+        for (int i = 0; i < m; ++i) c->hpos[b].push_back((int32_t)(c->cursor[b] + i));
+        c->live[b] += m;
+        c->cursor[b] += m;
+    }
+}
+
+}  // namespace
+
+extern "C" kvm_status kvm_kv_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sb, const int32_t* se,
+                                     int32_t* gather_out, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    return do_compact(c, span_cu, sb, se, gather_out, (cudaStream_t)stream);
+}
+
+extern "C" kvm_status kvm_tail_attn_prefill(kvm_ctx* c, int32_t layer, const int32_t* tail_cu, const void* q,
+                                            const void* k_new, const void* v_new, void* out, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    return do_attention(c, layer, tail_cu, q, k_new, v_new, out, (cudaStream_t)stream);
+}
+
+extern "C" kvm_status kvm_gdn_chunk_scan_from_state(kvm_ctx* c, int32_t layer, const int32_t* tail_cu,
+                                                    const void* q, const void* k, const void* v,
+                                                    const float* alpha, const float* beta, void* out,
+                                                    void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    return do_gdn(c, layer, tail_cu, q, k, v, alpha, beta, out, (cudaStream_t)stream);
+}
+
+extern "C" kvm_status kvm_advance(kvm_ctx* c, const int32_t* tail_cu) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    int total = 0;
+    kvm_status st = check_tail_cu(c, tail_cu, &total);
+    if (st) return st;
+    for (int b = 0; b < c->B; ++b)
+        if (c->live[b] + tail_cu[b + 1] - tail_cu[b] > c->cap[b])
+            return fail(KVM_E_CAPACITY, "character %d would exceed its capacity", b);
+    do_advance(c, tail_cu);
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* stream) {
+    if (!c || !r) return fail(KVM_E_INVAL, "NULL argument");
+    cudaStream_t s = (cudaStream_t)stream;
+    int total = 0;
+    kvm_status st = check_tail_cu(c, r->tail_cu, &total);
+    if (st) return st;
+    if (!r->q || !r->k || !r->v || !r->out) return fail(KVM_E_INVAL, "NULL per-layer pointer array");
+    // validate everything before the first launch: spans and capacity after removal
+    {
+        SpanPlan pl;
+        st = plan_spans(c, r->span_cu, r->span_begin, r->span_end, pl);
+        if (st) return st;
+        for (int b = 0; b < c->B; ++b) {
+            const int m = r->tail_cu[b + 1] - r->tail_cu[b];
+            if (pl.L_new[b] + m > c->cap[b])
+                return fail(KVM_E_CAPACITY, "character %d: live %d + tail %d exceeds capacity %d", b, pl.L_new[b],
+                            m, c->cap[b]);
+        }
+        for (int l = 0; l < c->n_layers; ++l) {
+            if (total > 0 && (!r->q[l] || !r->k[l] || !r->v[l] || !r->out[l]))
+                return fail(KVM_E_INVAL, "layer %d has a NULL tensor", l);
+            if (c->kind[l] == KVM_LAYER_GDN && total > 0 && (!r->alpha || !r->beta || !r->alpha[l] || !r->beta[l]))
+                return fail(KVM_E_INVAL, "layer %d has NULL gates", l);
+        }
+    }
+    st = do_compact(c, r->span_cu, r->span_begin, r->span_end, r->gather_out, s);
+    if (st) return st;
+    for (int l = 0; l < c->n_layers; ++l) {
+        const bool attn = c->kind[l] == KVM_LAYER_ATTN;
+        const size_t nq = (size_t)total * (attn ? c->Hq * c->D : c->H * c->dk) * 2;
+        const size_t nk = (size_t)total * (attn ? c->Hkv * c->D : c->H * c->dk) * 2;
+        const size_t nv = (size_t)total * (attn ? c->Hkv * c->D : c->H * c->dv) * 2;
+        const size_t ng = (size_t)total * c->H * 4;
+        const size_t no = (size_t)total * (attn ? c->Hq * c->D : c->H * c->dv) * 2;
+        const void *q = r->q[l], *k = r->k[l], *v = r->v[l];
+        const float *al = attn ? nullptr : r->alpha[l], *be = attn ? nullptr : r->beta[l];
+        void* out = r->out[l];
+        if (r->io_on_host && total > 0) {
+            CUDA_TRY(cudaMemcpyAsync(c->stage_in[0], q, nq, cudaMemcpyHostToDevice, s));
+            CUDA_TRY(cudaMemcpyAsync(c->stage_in[1], k, nk, cudaMemcpyHostToDevice, s));
+            CUDA_TRY(cudaMemcpyAsync(c->stage_in[2], v, nv, cudaMemcpyHostToDevice, s));
+            q = c->stage_in[0]; k = c->stage_in[1]; v = c->stage_in[2];
+            if (!attn) {
+                CUDA_TRY(cudaMemcpyAsync(c->stage_in[3], al, ng, cudaMemcpyHostToDevice, s));
+                CUDA_TRY(cudaMemcpyAsync(c->stage_in[4], be, ng, cudaMemcpyHostToDevice, s));
+                al = static_cast<const float*>(c->stage_in[3]);
+                be = static_cast<const float*>(c->stage_in[4]);
+            }
+            out = c->stage_out;
+        }
+        st = attn ? do_attention(c, l, r->tail_cu, q, k, v, out, s)
+                  : do_gdn(c, l, r->tail_cu, q, k, v, al, be, out, s);
+        if (st) return st;
+        if (r->io_on_host && total > 0)
+            CUDA_TRY(cudaMemcpyAsync(r->out[l], c->stage_out, no, cudaMemcpyDeviceToHost, s));
+    }
+    do_advance(c, r->tail_cu);
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_check(kvm_ctx* c, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    CUDA_TRY(cudaStreamSynchronize((cudaStream_t)stream));
+    int32_t e = 0;
+    CUDA_TRY(cudaMemcpy(&e, c->err, 4, cudaMemcpyDeviceToHost));
+    if (e) {
+        CUDA_TRY(cudaMemset(c->err, 0, 4));
+        CUDA_TRY(cudaMemset(c->tickets, 0, sizeof(int32_t) * (size_t)c->B * (2 * c->n_attn * c->Hkv + 1)));
+        return fail(KVM_E_DEVICE, "device error word 0x%x (%s%s)", e, (e & kErrBounds) ? "bounds " : "",
+                    (e & kErrWait) ? "wait-timeout" : "");
+    }
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_fork(kvm_ctx* dst, const kvm_ctx* src, void* stream) {
+    if (!dst || !src) return fail(KVM_E_INVAL, "NULL context");
+    if (dst == src) return KVM_OK;
+    if (dst->kind != src->kind || dst->Hq != src->Hq || dst->Hkv != src->Hkv || dst->D != src->D ||
+        dst->R != src->R || dst->theta != src->theta || dst->H != src->H || dst->dk != src->dk ||
+        dst->dv != src->dv || dst->B != src->B || dst->cap != src->cap)
+        return fail(KVM_E_INVAL, "contexts differ in model shape, population or capacity");
+    cudaStream_t s = (cudaStream_t)stream;
+    const size_t kv = (size_t)src->n_attn * src->Hkv * src->T_cap * src->D * sizeof(__nv_bfloat16);
+    if (kv) {
+        CUDA_TRY(cudaMemcpyAsync(dst->K, src->K, kv, cudaMemcpyDeviceToDevice, s));
+        CUDA_TRY(cudaMemcpyAsync(dst->V, src->V, kv, cudaMemcpyDeviceToDevice, s));
+        CUDA_TRY(cudaMemcpyAsync(dst->pos, src->pos, (size_t)src->T_cap * 4, cudaMemcpyDeviceToDevice, s));
+    }
+    const size_t sn = (size_t)src->n_gdn * src->B * src->H * src->dv * src->dk * sizeof(float);
+    if (sn) CUDA_TRY(cudaMemcpyAsync(dst->S, src->S, sn, cudaMemcpyDeviceToDevice, s));
+    dst->live = src->live;
+    dst->cursor = src->cursor;
+    dst->hpos = src->hpos;
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_profile_enable(kvm_ctx* c, int32_t enable) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (enable && c->ev.empty()) {
+        c->ev.resize(2 * kProfPool);
+        for (auto& e : c->ev) CUDA_TRY(cudaEventCreate(&e));
+    }
+    c->prof = enable != 0;
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_profile_read(kvm_ctx* c, int32_t kernel, int64_t* launches, double* total_ms,
+                                       int32_t reset) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (kernel < 0 || kernel >= KVM_K_COUNT) return fail(KVM_E_INVAL, "kernel family %d out of range", kernel);
+    CUDA_TRY(cudaDeviceSynchronize());
+    double ms = 0.0;
+    for (size_t i = 0; i < c->ev_kind.size(); ++i) {
+        if (c->ev_kind[i] != kernel) continue;
+        float t = 0.f;
+        CUDA_TRY(cudaEventElapsedTime(&t, c->ev[2 * i], c->ev[2 * i + 1]));
+        ms += t;
+    }
+    if (launches) *launches = c->prof_launches[kernel];
+    if (total_ms) *total_ms = ms;
+    if (reset) {
+        c->ev_kind.clear();
+        for (auto& n : c->prof_launches) n = 0;
+    }
+    return KVM_OK;
+}

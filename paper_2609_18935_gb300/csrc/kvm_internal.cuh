@@ -1,0 +1,138 @@
+// Internal declarations of the maintenance library (kernels + host runtime).
+// Everything here is private to libkvm; the public ABI is include/kvm.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+namespace kvm {
+
+constexpr int kMaxChars = 256;      // characters per context (per-round descriptors travel as kernel parameters)
+constexpr int kMaxSpans = 1024;     // deletion spans per round, all characters together
+constexpr int kMaxRotaryHalf = 128; // rotary_dim / 2
+
+// Device error word bits (read by kvm_check).
+constexpr int kErrBounds = 1;       // an index fell outside the buffers a kernel was given
+constexpr int kErrWait = 2;         // a bounded wait expired
+
+// ----------------------------------------------------------------------------
+// kv_compact
+// ----------------------------------------------------------------------------
+constexpr int kCompactThreads = 256;
+constexpr int kCompactVecPerThread = 4;            // 16-byte vectors held per thread
+constexpr int kCompactVecPerChunk = kCompactThreads * kCompactVecPerThread;
+
+struct CompactChar {
+    int32_t L_new;        // live length after removal
+    int32_t first;        // first removed live index (= first moved destination)
+    int32_t seg_off;      // offset of this character's segments in seg_start/seg_shift
+    int32_t n_seg;        // number of spans (= moved segments)
+    int32_t cap_off;      // slot offset of the character inside every slab
+    int32_t chunks_kv;    // chunks per KV slab
+    int32_t chunks_pos;   // chunks of the position slab
+    int32_t blk_off;      // first block of this character
+    int32_t flag_off;     // first read-flag of this character
+};
+
+struct CompactParams {
+    int32_t n_chars;
+    int32_t n_kv_slabs;   // 2 * n_attn * n_kv_heads  (K slabs, then V slabs)
+    int32_t vec_per_row;  // 16-byte vectors per KV row (head_dim * 2 / 16)
+    int32_t rows_kv;      // rows per KV chunk
+    int32_t rows_pos;     // rows per position chunk
+    int32_t total_blocks;
+    uint32_t epoch;
+    int64_t slab_rows;    // rows per (layer, head) slab = total capacity
+    uint4* K;
+    uint4* V;
+    int32_t* pos;
+    int32_t* tickets;     // [n_chars][n_kv_slabs + 1]
+    uint32_t* flags;
+    int32_t* err;
+    CompactChar ch[kMaxChars];
+    // segment k of a character: survivors whose new index is >= seg_start[k]
+    // (and below the next segment's start) come from new index + seg_shift[k]
+    int32_t seg_start[kMaxSpans];
+    int32_t seg_shift[kMaxSpans];
+};
+
+void launch_kv_compact(const CompactParams& p, cudaStream_t s);
+
+struct GatherParams {
+    int32_t n_chars;
+    int32_t total;        // sum of L_new
+    int32_t out_off[kMaxChars + 1];
+    int32_t first[kMaxChars];
+    int32_t seg_off[kMaxChars];
+    int32_t n_seg[kMaxChars];
+    int32_t* out;
+    int32_t seg_start[kMaxSpans];
+    int32_t seg_shift[kMaxSpans];
+};
+void launch_gather_map(const GatherParams& p, cudaStream_t s);
+
+// ----------------------------------------------------------------------------
+// tail attention
+// ----------------------------------------------------------------------------
+struct AttnChar {
+    int32_t L_prev;       // surviving live entries (L')
+    int32_t M;            // tail tokens
+    int32_t tail_off;     // first packed tail row
+    int32_t cap_off;      // slot offset of the character in the slabs
+    int64_t p;            // cursor: position of tail token 0
+    int32_t n_qtiles;     // query tiles per KV head
+    int32_t item_off;     // first work item (tile * split) of this character
+};
+
+struct AttnParams {
+    int32_t n_chars;
+    int32_t Hq, Hkv, D, R, g;
+    int32_t n_split;      // key splits per query tile
+    int32_t n_items;      // total work items
+    int32_t tok_per_tile; // tail tokens per 64-row query tile (64 / g)
+    float scale_log2;     // log2(e) / sqrt(D)
+    int64_t slab_rows;    // rows per (layer, head) slab
+    const __nv_bfloat16* q;       // caller's unrotated q  [sum M][Hq][D]
+    const __nv_bfloat16* k_new;   // [sum M][Hkv][D]
+    const __nv_bfloat16* v_new;
+    __nv_bfloat16* q_rot;         // workspace [sum M][Hq][D]
+    __nv_bfloat16* K;             // this layer's K slabs [Hkv][slab_rows][D]
+    __nv_bfloat16* V;
+    int32_t* pos;                 // [slab_rows]
+    __nv_bfloat16* out;           // [sum M][Hq][D]
+    float* part_o;                // [n_items][64][D]
+    float* part_ml;               // [n_items][64][2]
+    int32_t* err;
+    double inv_freq[kMaxRotaryHalf];
+    AttnChar ch[kMaxChars];
+};
+
+void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s);
+void launch_tail_attention(const AttnParams& p, cudaStream_t s);
+void launch_attn_combine(const AttnParams& p, int n_tiles, cudaStream_t s);
+
+// ----------------------------------------------------------------------------
+// gated delta rule
+// ----------------------------------------------------------------------------
+struct GdnChar {
+    int32_t M;
+    int32_t tail_off;
+};
+
+struct GdnParams {
+    int32_t n_chars, H, dk, dv;
+    const __nv_bfloat16* q;   // [sum M][H][dk]
+    const __nv_bfloat16* k;
+    const __nv_bfloat16* v;   // [sum M][H][dv]
+    const float* alpha;       // [sum M][H]
+    const float* beta;
+    __nv_bfloat16* out;       // [sum M][H][dv]
+    float* S;                 // this layer's state [n_chars][H][dv][dk]
+    int32_t* err;
+    GdnChar ch[kMaxChars];
+};
+
+void launch_gdn_chunk_scan(const GdnParams& p, cudaStream_t s);
+
+}  // namespace kvm

@@ -1,0 +1,281 @@
+"""Thin Python binding of libkvm (include/kvm.h).
+
+Argument marshalling only: every step of the maintenance path runs in the
+library's CUDA kernels.  Tensors are torch CUDA tensors (device memory and
+streams come from PyTorch); host-side index arrays are numpy int32/int64.
+The binding has no fallback: if libkvm.so has not been built, loading it
+raises immediately.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.environ.get("KVM_LIB", os.path.join(_PKG, "_build", "libkvm.so"))
+
+KVM_OK, KVM_E_INVAL, KVM_E_SPAN, KVM_E_CAPACITY, KVM_E_CUDA, KVM_E_DEVICE, KVM_E_UNSUPPORTED = range(7)
+LAYER_GDN, LAYER_ATTN = 0, 1
+
+_ERRNAMES = {1: "KVM_E_INVAL", 2: "KVM_E_SPAN", 3: "KVM_E_CAPACITY", 4: "KVM_E_CUDA",
+             5: "KVM_E_DEVICE", 6: "KVM_E_UNSUPPORTED"}
+
+
+class KvmError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{_ERRNAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+class ModelDesc(C.Structure):
+    _fields_ = [("n_layers", C.c_int32), ("layer_kind", C.POINTER(C.c_int32)),
+                ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32), ("head_dim", C.c_int32),
+                ("rotary_dim", C.c_int32), ("rope_theta", C.c_double), ("n_gdn_heads", C.c_int32),
+                ("d_k", C.c_int32), ("d_v", C.c_int32)]
+
+
+class Round(C.Structure):
+    _fields_ = [("span_cu", C.POINTER(C.c_int32)), ("span_begin", C.POINTER(C.c_int32)),
+                ("span_end", C.POINTER(C.c_int32)), ("tail_cu", C.POINTER(C.c_int32)),
+                ("q", C.POINTER(C.c_void_p)), ("k", C.POINTER(C.c_void_p)), ("v", C.POINTER(C.c_void_p)),
+                ("alpha", C.POINTER(C.c_void_p)), ("beta", C.POINTER(C.c_void_p)),
+                ("out", C.POINTER(C.c_void_p)), ("io_on_host", C.c_int32),
+                ("gather_out", C.c_void_p)]
+
+
+# name -> (restype, argtypes)
+_SIGS = {
+    "kvm_create": (C.c_int, [C.POINTER(ModelDesc), C.c_int32, C.POINTER(C.c_int32), C.c_int32,
+                             C.POINTER(C.c_void_p)]),
+    "kvm_destroy": (C.c_int, [C.c_void_p]),
+    "kvm_last_error": (C.c_char_p, []),
+    "kvm_load_prefix": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int64, C.POINTER(C.c_int32),
+                                  C.c_void_p]),
+    "kvm_set_kv": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "kvm_get_kv": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "kvm_get_positions": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "kvm_set_state": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "kvm_get_state": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "kvm_get_live": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int64)]),
+    "kvm_spans_from_positions": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.POINTER(C.c_int64),
+                                           C.POINTER(C.c_int64), C.POINTER(C.c_int32),
+                                           C.POINTER(C.c_int32)]),
+    "kvm_kv_compact": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.POINTER(C.c_int32),
+                                 C.POINTER(C.c_int32), C.c_void_p, C.c_void_p]),
+    "kvm_tail_attn_prefill": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int32), C.c_void_p,
+                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "kvm_gdn_chunk_scan_from_state": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int32), C.c_void_p,
+                                                C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                                C.c_void_p, C.c_void_p]),
+    "kvm_advance": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32)]),
+    "kvm_update_round": (C.c_int, [C.c_void_p, C.POINTER(Round), C.c_void_p]),
+    "kvm_check": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "kvm_launch_count": (C.c_int64, [C.c_void_p]),
+    "kvm_fork": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "kvm_profile_enable": (C.c_int, [C.c_void_p, C.c_int32]),
+    "kvm_profile_read": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double),
+                                   C.c_int32]),
+}
+
+# kernel families of kvm_profile_read
+K_COMPACT, K_ROPE_APPEND, K_ATTENTION, K_ATTN_COMBINE, K_GDN, K_GATHER = range(6)
+KERNEL_NAMES = ["kv_compact", "rope_append", "tail_attention", "attn_combine", "gdn_chunk_scan", "gather_map"]
+
+_lib = None
+
+
+def load_library(path: str | None = None):
+    """Load libkvm.so once; raises OSError if it is missing (no fallback)."""
+    global _lib
+    if _lib is None:
+        p = path or LIB_PATH
+        if not os.path.exists(p):
+            raise OSError(f"libkvm.so not found at {p}; build it with "
+                          "`python -m paper_2609_18935_gb300.build_lib`")
+        lib = C.CDLL(p)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+    return _lib
+
+
+def _check(status: int):
+    if status != KVM_OK:
+        raise KvmError(status, _lib.kvm_last_error().decode())
+
+
+def _i32(a) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+
+
+def _p32(a: np.ndarray):
+    return a.ctypes.data_as(C.POINTER(C.c_int32))
+
+
+def _dptr(t, dtype=None) -> int:
+    """Device address of a contiguous torch CUDA tensor (0 for None)."""
+    if t is None:
+        return 0
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"expected {dtype}, got {t.dtype}")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+class Context:
+    """A population of character states on the current CUDA device (kvm_create)."""
+
+    def __init__(self, layer_kind, n_q_heads, n_kv_heads, head_dim, rotary_dim, rope_theta,
+                 n_gdn_heads, d_k, d_v, capacity, max_tail_tokens):
+        lib = load_library()
+        self.layer_kind = [int(x) for x in layer_kind]
+        self._kinds = _i32(self.layer_kind)
+        self.desc = ModelDesc(len(self.layer_kind), _p32(self._kinds), n_q_heads, n_kv_heads, head_dim,
+                              rotary_dim, float(rope_theta), n_gdn_heads, d_k, d_v)
+        self.n_chars = len(capacity)
+        self.Hq, self.Hkv, self.D, self.R = n_q_heads, n_kv_heads, head_dim, rotary_dim
+        self.H, self.dk, self.dv = n_gdn_heads, d_k, d_v
+        caps = _i32(capacity)
+        h = C.c_void_p()
+        _check(lib.kvm_create(C.byref(self.desc), self.n_chars, _p32(caps), int(max_tail_tokens), C.byref(h)))
+        self._h = h
+
+    def destroy(self):
+        if self._h:
+            _check(_lib.kvm_destroy(self._h))
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+    # ---------------------------------------------------------------- state
+    def load_prefix(self, b, live, cursor, positions, stream=None):
+        pos = _i32(positions)
+        _check(_lib.kvm_load_prefix(self._h, b, int(live), int(cursor), _p32(pos), _stream(stream)))
+
+    def set_kv(self, layer, b, k, v, stream=None):
+        import torch
+        _check(_lib.kvm_set_kv(self._h, layer, b, _dptr(k, torch.bfloat16), _dptr(v, torch.bfloat16),
+                               _stream(stream)))
+
+    def get_kv(self, layer, b, stream=None):
+        import torch
+        live, _ = self.get_live(b)
+        k = torch.empty((self.Hkv, live, self.D), dtype=torch.bfloat16, device="cuda")
+        v = torch.empty_like(k)
+        _check(_lib.kvm_get_kv(self._h, layer, b, _dptr(k), _dptr(v), _stream(stream)))
+        return k, v
+
+    def get_positions(self, b, stream=None):
+        import torch
+        live, _ = self.get_live(b)
+        out = torch.empty(live, dtype=torch.int32, device="cuda")
+        _check(_lib.kvm_get_positions(self._h, b, _dptr(out), _stream(stream)))
+        return out
+
+    def set_state(self, layer, S, stream=None):
+        import torch
+        _check(_lib.kvm_set_state(self._h, layer, _dptr(S, torch.float32), _stream(stream)))
+
+    def get_state(self, layer, stream=None):
+        import torch
+        S = torch.empty((self.n_chars, self.H, self.dv, self.dk), dtype=torch.float32, device="cuda")
+        _check(_lib.kvm_get_state(self._h, layer, _dptr(S), _stream(stream)))
+        return S
+
+    def get_live(self, b):
+        live, cur = C.c_int32(), C.c_int64()
+        _check(_lib.kvm_get_live(self._h, b, C.byref(live), C.byref(cur)))
+        return live.value, cur.value
+
+    def spans_from_positions(self, b, pos_begin, pos_end):
+        pb = np.ascontiguousarray(pos_begin, dtype=np.int64)
+        pe = np.ascontiguousarray(pos_end, dtype=np.int64)
+        n = len(pb)
+        sb = np.zeros(n, np.int32)
+        se = np.zeros(n, np.int32)
+        _check(_lib.kvm_spans_from_positions(self._h, b, n, pb.ctypes.data_as(C.POINTER(C.c_int64)),
+                                             pe.ctypes.data_as(C.POINTER(C.c_int64)), _p32(sb), _p32(se)))
+        return sb, se
+
+    # ---------------------------------------------------------------- hot path
+    def kv_compact(self, span_cu, span_begin, span_end, gather_out=None, stream=None):
+        import torch
+        cu, sb, se = _i32(span_cu), _i32(span_begin), _i32(span_end)
+        _check(_lib.kvm_kv_compact(self._h, _p32(cu), _p32(sb), _p32(se), _dptr(gather_out, torch.int32),
+                                   _stream(stream)))
+
+    def tail_attn_prefill(self, layer, tail_cu, q, k_new, v_new, out, stream=None):
+        import torch
+        cu = _i32(tail_cu)
+        bf = torch.bfloat16
+        _check(_lib.kvm_tail_attn_prefill(self._h, layer, _p32(cu), _dptr(q, bf), _dptr(k_new, bf),
+                                          _dptr(v_new, bf), _dptr(out, bf), _stream(stream)))
+
+    def gdn_chunk_scan_from_state(self, layer, tail_cu, q, k, v, alpha, beta, out, stream=None):
+        import torch
+        cu = _i32(tail_cu)
+        bf, f = torch.bfloat16, torch.float32
+        _check(_lib.kvm_gdn_chunk_scan_from_state(self._h, layer, _p32(cu), _dptr(q, bf), _dptr(k, bf),
+                                                  _dptr(v, bf), _dptr(alpha, f), _dptr(beta, f),
+                                                  _dptr(out, bf), _stream(stream)))
+
+    def advance(self, tail_cu):
+        cu = _i32(tail_cu)
+        _check(_lib.kvm_advance(self._h, _p32(cu)))
+
+    def update_round(self, span_cu, span_begin, span_end, tail_cu, inputs, outputs,
+                     io_on_host=False, gather_out=None, stream=None):
+        """One whole round (kvm_update_round).
+
+        inputs[layer] = dict(q, k, v[, alpha, beta]) and outputs[layer] = tensor,
+        CUDA tensors (io_on_host=False) or pinned CPU tensors (io_on_host=True)."""
+        n = len(self.layer_kind)
+        arr = lambda: (C.c_void_p * n)()
+        q, k, v, al, be, out = arr(), arr(), arr(), arr(), arr(), arr()
+        ptr = (lambda t: t.data_ptr() if t is not None else 0)
+        for l in range(n):
+            x = inputs[l]
+            q[l], k[l], v[l] = ptr(x["q"]), ptr(x["k"]), ptr(x["v"])
+            al[l], be[l] = ptr(x.get("alpha")), ptr(x.get("beta"))
+            out[l] = ptr(outputs[l])
+        cu, sb, se, tc = _i32(span_cu), _i32(span_begin), _i32(span_end), _i32(tail_cu)
+        r = Round(_p32(cu), _p32(sb), _p32(se), _p32(tc), q, k, v, al, be, out, int(bool(io_on_host)),
+                  ptr(gather_out))
+        self._keep = (cu, sb, se, tc, q, k, v, al, be, out)
+        _check(_lib.kvm_update_round(self._h, C.byref(r), _stream(stream)))
+
+    def check(self, stream=None):
+        _check(_lib.kvm_check(self._h, _stream(stream)))
+
+    def launch_count(self) -> int:
+        return int(_lib.kvm_launch_count(self._h))
+
+    def fork_from(self, src: "Context", stream=None):
+        """Overwrite this context's state with a copy of `src` (kvm_fork)."""
+        _check(_lib.kvm_fork(self._h, src._h, _stream(stream)))
+
+    def profile_enable(self, enable=True):
+        _check(_lib.kvm_profile_enable(self._h, int(bool(enable))))
+
+    def profile_read(self, kernel, reset=False):
+        """(launches, total device ms) of one kernel family since the last reset."""
+        n, ms = C.c_int64(), C.c_double()
+        _check(_lib.kvm_profile_read(self._h, kernel, C.byref(n), C.byref(ms), int(bool(reset))))
+        return n.value, ms.value

@@ -1,0 +1,155 @@
+"""GPU parity: the CUDA library (through its C ABI) against the fp64 oracle.
+
+Bar: compaction indices, cache bytes and positions bit-exact; attention
+outputs, delta-rule outputs and carried states within relative L2 5e-3 of the
+oracle (bf16 inputs, fp32 accumulation), after every round of a chain.
+"""
+import numpy as np
+import pytest
+
+from workload import synth as W
+
+pytestmark = pytest.mark.gpu
+
+TOL = 5e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_18935_gb300 import kvm
+    kvm.load_library()
+
+
+def _assert_errs(errs, tol=TOL, what=""):
+    bad = {k: v for k, v in errs.items() if not (v <= tol)}
+    assert not bad, f"{what} rel-L2 above {tol}: {bad}"
+
+
+def test_tiny_round_matches_oracle():
+    from harness import Pair
+    w = W.make_workload("tiny")
+    pair = Pair(w.shape, w.prefix_len, w.capacity(), 64, seed_index=w.index, prefix="refill")
+    live = [pair.ctx.get_live(0)[0]]
+    span_cu, sb, se, tails = W.round_plan(w, 0, live)
+    assert int((se - sb).sum()) == 64 and len(sb) == 2
+    errs = pair.run_round(span_cu, sb, se, tails, W.tail_inputs(w, 0, tails))
+    _assert_errs(errs, what="tiny")
+
+
+def test_tiny_round_via_separate_entry_points():
+    from harness import Pair
+    w = W.make_workload("tiny")
+    pair = Pair(w.shape, w.prefix_len, w.capacity(), 64, seed_index=w.index, prefix="refill")
+    span_cu, sb, se, tails = W.round_plan(w, 0, [512])
+    errs = pair.run_round(span_cu, sb, se, tails, W.tail_inputs(w, 0, tails), via="entry_points")
+    _assert_errs(errs, what="tiny/entry points")
+
+
+def test_npc_shape_eight_chained_rounds():
+    """NPC-shaped stack (D 256, 16/2 heads, delta d 128, 3:1), shorter prefix so
+    the oracle keeps up; 8 chained rounds, ragged tail (96 tokens: 1.5 chunks,
+    12 query tiles)."""
+    from harness import Pair
+    shape = W.npc_shape(4)
+    N, M = 1024, 96
+    w = W.Workload("npc-small", 11, shape, [N], 8)
+    w.plan = [[(0.05, 1 + r % 4, M)] for r in range(8)]
+    pair = Pair(shape, [N], w.capacity(), M, seed_index=w.index)
+    for r in range(8):
+        live = [pair.ctx.get_live(0)[0]]
+        span_cu, sb, se, tails = W.round_plan(w, r, live)
+        errs = pair.run_round(span_cu, sb, se, tails, W.tail_inputs(w, r, tails))
+        _assert_errs(errs, what=f"round {r}")
+
+
+def test_population_varlen_edge_cases():
+    """Several characters packed: a character with nothing removed, one whose
+    whole cache is removed (the tail attends to itself only), one with no tail
+    this round, spans at the very start and end, tails of 1 and 130 tokens."""
+    from harness import Pair
+    shape = W.ModelShape([W.GDN, W.ATTN, W.GDN, W.ATTN], 8, 2, 128, 64, 1e4, 4, 64, 96)
+    prefix = [300, 64, 517, 129, 40]
+    caps = [640, 256, 768, 384, 256]
+    pair = Pair(shape, prefix, caps, 512, seed_index=21)
+    spans = {0: ([], []), 1: ([0], [64]), 2: ([0, 100, 510], [3, 300, 517]), 3: ([5], [6]), 4: ([39], [40])}
+    tails = [70, 33, 1, 0, 130]
+    cu, sb, se = [0], [], []
+    for b in range(5):
+        sb += spans[b][0]
+        se += spans[b][1]
+        cu.append(len(sb))
+    w = W.Workload("edge", 21, shape, prefix, 1)
+    w.plan = [[(0, 0, m) for m in tails]]
+    ins = W.tail_inputs(w, 0, tails)
+    errs = pair.run_round(np.array(cu, np.int32), np.array(sb, np.int32), np.array(se, np.int32), tails, ins)
+    _assert_errs(errs, what="edge")
+    # a second round on the same population (earlier tails become removable)
+    spans2 = [([0], [10]), ([2], [30]), ([100], [200]), ([0], [128]), ([0], [1])]
+    cu, sb, se = [0], [], []
+    for b in range(5):
+        sb += spans2[b][0]
+        se += spans2[b][1]
+        cu.append(len(sb))
+    tails2 = [64, 64, 64, 64, 64]
+    w.plan = [[(0, 0, m) for m in tails2]]
+    errs = pair.run_round(np.array(cu, np.int32), np.array(sb, np.int32), np.array(se, np.int32), tails2,
+                          W.tail_inputs(w, 0, tails2))
+    _assert_errs(errs, what="edge round 2")
+
+
+def test_large_cursor_positions():
+    """Positions far beyond the live length (holes only in position space)."""
+    from harness import Pair
+    shape = W.ModelShape([W.ATTN], 16, 2, 256, 64, 1e4, 1, 64, 32)
+    pair = Pair(shape, [200], [512], 64, seed_index=31, cursor_offset=479_000)
+    w = W.Workload("far", 31, shape, [200], 1)
+    w.plan = [[(0.1, 3, 64)]]
+    span_cu, sb, se, tails = W.round_plan(w, 0, [200])
+    errs = pair.run_round(span_cu, sb, se, tails, W.tail_inputs(w, 0, tails))
+    _assert_errs(errs, what="far positions")
+
+
+def test_rejected_calls_leave_state_unchanged():
+    import torch
+    from harness import Pair
+    from paper_2609_18935_gb300 import kvm
+    shape = W.TINY
+    pair = Pair(shape, [100], [256], 64, seed_index=41)
+    before = pair.snapshot_kv()
+    S_before = pair.ctx.get_state(0).cpu()
+    bad = [([0, 2], [30, 10], [20, 40]),    # overlap
+           ([0, 1], [50], [50]),            # empty
+           ([0, 1], [90], [101]),           # outside live
+           ([0, 2], [40, 10], [50, 20])]    # unsorted
+    for cu, b, e in bad:
+        with pytest.raises(kvm.KvmError) as ei:
+            pair.ctx.kv_compact(np.array(cu), np.array(b), np.array(e))
+        assert ei.value.code == kvm.KVM_E_SPAN
+    q = torch.zeros((200, 8, 64), dtype=torch.bfloat16, device="cuda")
+    kv = torch.zeros((200, 2, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(kvm.KvmError) as ei:     # 100 live + 200 > capacity 256
+        pair.ctx.tail_attn_prefill(1, np.array([0, 200]), q, kv, kv, q)
+    assert ei.value.code == kvm.KVM_E_CAPACITY
+    with pytest.raises(kvm.KvmError) as ei:     # wrong layer kind
+        pair.ctx.tail_attn_prefill(0, np.array([0, 10]), q, kv, kv, q)
+    assert ei.value.code == kvm.KVM_E_INVAL
+    pair.ctx.check()
+    after = pair.snapshot_kv()
+    for key in before:
+        for x, y in zip(before[key], after[key]):
+            assert np.array_equal(x, y)
+    assert torch.equal(S_before, pair.ctx.get_state(0).cpu())
+    assert pair.ctx.get_live(0) == (100, 100)
+
+
+def test_spans_from_positions():
+    from harness import Pair
+    from paper_2609_18935_gb300 import kvm
+    pair = Pair(W.TINY, [50], [256], 64, seed_index=51, cursor_offset=1000)
+    sb, se = pair.ctx.spans_from_positions(0, [1005, 1040], [1010, 1041])
+    assert list(sb) == [5, 40] and list(se) == [10, 41]
+    with pytest.raises(kvm.KvmError):
+        pair.ctx.spans_from_positions(0, [0], [10])     # covers no live entry

@@ -300,3 +300,50 @@ def prefix_cache(w: Workload, b: int, layer: int, n: int):
 def prefix_state(w: Workload, b: int, layer: int) -> np.ndarray:
     s = w.shape
     return state_f32((w.index * 1000 + 997, b, layer), (s.n_gdn_heads, s.d_v, s.d_k))
+
+
+# ----------------------------------------------------------------------------
+# device-side draws (benchmark inputs too large to draw on the CPU quickly)
+# ----------------------------------------------------------------------------
+def device_round_inputs(w: Workload, seed: int, tails: list, device="cuda") -> dict:
+    """Same distributions as `tail_inputs`, drawn on the GPU with a seeded
+    torch generator (not bit-identical to the numpy draws).  Returns
+    {layer: dict of torch tensors} packed over characters."""
+    import torch
+    s = w.shape
+    total = int(sum(tails))
+    g = torch.Generator(device=device)
+    out = {}
+    for layer, kind in enumerate(s.layer_kind):
+        g.manual_seed(int(seed) * 1009 + layer)
+        if kind == ATTN:
+            q = torch.randn((total, s.n_q_heads, s.head_dim), generator=g, device=device)
+            k = torch.randn((total, s.n_kv_heads, s.head_dim), generator=g, device=device)
+            v = torch.randn((total, s.n_kv_heads, s.head_dim), generator=g, device=device)
+            d = {}
+        else:
+            q = torch.randn((total, s.n_gdn_heads, s.d_k), generator=g, device=device)
+            k = torch.randn((total, s.n_gdn_heads, s.d_k), generator=g, device=device)
+            v = torch.randn((total, s.n_gdn_heads, s.d_v), generator=g, device=device)
+            a = torch.sigmoid(3.0 + 0.5 * torch.randn((total, s.n_gdn_heads), generator=g, device=device))
+            bt = torch.sigmoid(torch.randn((total, s.n_gdn_heads), generator=g, device=device))
+            d = {"alpha": a.float().contiguous(), "beta": bt.float().contiguous()}
+        k = k / k.norm(dim=-1, keepdim=True)
+        d.update({"q": q.bfloat16().contiguous(), "k": k.bfloat16().contiguous(),
+                  "v": v.bfloat16().contiguous()})
+        out[layer] = d
+    return out
+
+
+def simulate_plan(w: Workload):
+    """Spans and tails of every round of `w`, following live lengths from the
+    prefix: list of (span_cu, begins, ends, tails)."""
+    live = list(w.prefix_len)
+    plan = []
+    for r in range(w.rounds):
+        cu, bs, es, tails = round_plan(w, r, live)
+        plan.append((cu, bs, es, tails))
+        for b in range(w.n_chars):
+            removed = int((es[cu[b]:cu[b + 1]] - bs[cu[b]:cu[b + 1]]).sum())
+            live[b] = live[b] - removed + tails[b]
+    return plan
