@@ -213,6 +213,39 @@ typedef struct kvm_round {
 
 kvm_status kvm_update_round(kvm_ctx* ctx, const kvm_round* round, void* stream);
 
+/* Allocation-free compaction for callers that cannot call cudaMalloc --
+ * for example an engine that owns all device memory through its own fixed
+ * arena and forbids other allocations during a session, or a frame loop in
+ * which an allocation (which may synchronize the device) would stall the
+ * frame.  Such callers cannot create a context, so this call removes the
+ * given live-index spans from KV buffers they own, with the same in-place
+ * result as kvm_kv_compact.  The paper has no counterpart of this call.
+ * K, V: device [n_slabs][slab_rows][head_dim] bf16 (n_slabs = attention
+ * layers x KV heads, every slab loses the same rows); positions: device
+ * [slab_rows] int32, compacted too, or NULL.  live: rows in use before the
+ * call; spans: host [n_spans], sorted, disjoint, inside [0, live).
+ * new_live_out (host) receives live minus the removed rows.
+ * Scratch: the kernel's bookkeeping lives in a fixed ~260 KB device array
+ * inside the library (every GPU that loads the library holds it until the
+ * process exits); this call allocates nothing.  Limits: n_slabs <= 512,
+ * n_spans <= 1024, head_dim in {64, 128, 256}, and
+ * 2 * n_slabs * ceil(moved / (8192 / head_dim)) + ceil(moved / 1024) <= 65536
+ * where moved = rows from the first span to the new live end (e.g. 24 slabs
+ * of head_dim 256 allow ~43K moved rows); larger requests return
+ * KVM_E_CAPACITY.  The first call on each device looks up the array's device
+ * address (cudaGetSymbolAddress); make that first call before any stream
+ * capture.  Every call shares the one array and clears the part it uses, so
+ * calls that may overlap on the GPU (other streams, other host threads on
+ * the same device) race: order them.  A device-side wait that expires
+ * (which valid arguments never cause) leaves that chunk unmoved and sets a
+ * bit in the array's error word; this call does not read it back.
+ * Errors: KVM_E_INVAL, KVM_E_SPAN, KVM_E_CAPACITY, KVM_E_UNSUPPORTED,
+ * KVM_E_CUDA. */
+kvm_status kvm_kv_compact_noalloc(void* K, void* V, int32_t* positions, int32_t n_slabs,
+                                  int64_t slab_rows, int32_t head_dim, int32_t live,
+                                  int32_t n_spans, const int32_t* span_begin,
+                                  const int32_t* span_end, int32_t* new_live_out, void* stream);
+
 /* Copy the whole state of `src` into `dst`: every character's live KV,
  * positions, recurrent states, live lengths and cursors (§4.2: task-specific
  * continuations branch from a maintained root).  Both contexts must have the

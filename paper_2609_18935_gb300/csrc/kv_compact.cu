@@ -17,6 +17,8 @@
 // holds).  Blocks wait only on chunks with earlier tickets, which are
 // resident or finished, so the waits always end; each wait is still bounded
 // and reports kErrWait instead of spinning forever.
+#include <cstring>
+
 #include "kvm_internal.cuh"
 
 namespace kvm {
@@ -174,3 +176,134 @@ void launch_gather_map(const GatherParams& p, cudaStream_t s) {
 }
 
 }  // namespace kvm
+
+// ============================================================================
+// Allocation-free compaction of caller-owned KV slabs.
+//
+// For callers that cannot call cudaMalloc: for example a game engine that
+// owns all device memory through its own fixed arena and forbids other
+// allocations during a session, or a frame loop in which an allocation (which
+// may synchronize the device) would stall the frame.  Such callers cannot
+// create a kvm context (kvm_create allocates), so this entry point compacts
+// KV buffers they own, and keeps the few words of bookkeeping the kernel
+// needs (per-slab tickets, per-chunk read flags, an error word) in the
+// fixed-size device array below instead of allocated workspace.  That array
+// lives in every GPU that loads the library until the process exits.
+// ============================================================================
+#include "../../include/kvm.h"
+
+namespace {
+constexpr int kNoAllocMaxSlabs = 512;                       // K slabs (layers x KV heads), V slabs as many
+constexpr int kNoAllocTickets = 2 * kNoAllocMaxSlabs + 1;   // + the position slab
+constexpr int kNoAllocMaxFlags = 65536;                     // read flags (one per moved chunk per slab)
+constexpr int kNoAllocWords = 64 + kNoAllocTickets + kNoAllocMaxFlags;   // word 0: device error word
+constexpr int kMaxDevices = 64;
+}  // namespace
+
+static __device__ __align__(256) uint32_t kvm_noalloc_scratch[kNoAllocWords];
+
+namespace {
+// Device address of kvm_noalloc_scratch per device, found once per device
+// (the name is a host-side stand-in; only cudaGetSymbolAddress gives the
+// address a kernel can use).
+uint32_t* g_noalloc_addr[kMaxDevices] = {};
+}  // namespace
+
+extern "C" kvm_status kvm_kv_compact_noalloc(void* K, void* V, int32_t* positions, int32_t n_slabs,
+                                             int64_t slab_rows, int32_t head_dim, int32_t live,
+                                             int32_t n_spans, const int32_t* span_begin,
+                                             const int32_t* span_end, int32_t* new_live_out, void* stream) {
+    using namespace kvm;
+    if (!K || !V) return report_error(KVM_E_INVAL, "kv_compact_noalloc: K or V is NULL");
+    if (n_slabs <= 0 || n_slabs > kNoAllocMaxSlabs)
+        return report_error(KVM_E_CAPACITY, "kv_compact_noalloc: n_slabs must be in [1, 512]");
+    if (head_dim != 64 && head_dim != 128 && head_dim != 256)
+        return report_error(KVM_E_UNSUPPORTED, "kv_compact_noalloc: head_dim must be 64, 128 or 256");
+    if (live < 0 || slab_rows < live || slab_rows > INT32_MAX)
+        return report_error(KVM_E_INVAL, "kv_compact_noalloc: need 0 <= live <= slab_rows <= 2^31-1");
+    if (n_spans < 0 || n_spans > kMaxSpans)
+        return report_error(KVM_E_CAPACITY, "kv_compact_noalloc: n_spans must be in [0, 1024]");
+    if (n_spans > 0 && (!span_begin || !span_end))
+        return report_error(KVM_E_INVAL, "kv_compact_noalloc: span arrays are NULL");
+    if (!new_live_out) return report_error(KVM_E_INVAL, "kv_compact_noalloc: new_live_out is NULL");
+
+    thread_local static CompactParams p;
+    std::memset(&p, 0, sizeof p);
+    int removed = 0, prev_end = 0;
+    for (int k = 0; k < n_spans; ++k) {
+        const int lo = span_begin[k], hi = span_end[k];
+        if (!(0 <= lo && lo < hi && hi <= live))
+            return report_error(KVM_E_SPAN, "kv_compact_noalloc: span empty or outside the live rows");
+        if (k > 0 && lo < prev_end)
+            return report_error(KVM_E_SPAN, "kv_compact_noalloc: spans must be sorted and disjoint");
+        prev_end = hi;
+        removed += hi - lo;
+        p.seg_start[k] = hi - removed;
+        p.seg_shift[k] = removed;
+    }
+    const int L_new = live - removed;
+    const int vec_per_row = head_dim * 2 / 16;
+    const int rows_kv = kCompactVecPerChunk / vec_per_row;
+    const int rows_pos = kCompactVecPerChunk;
+    const int moved = n_spans > 0 ? L_new - span_begin[0] : 0;
+    const int chunks_kv = (moved + rows_kv - 1) / rows_kv;
+    const int chunks_pos = positions ? (moved + rows_pos - 1) / rows_pos : 0;
+    const int64_t n_flags = (int64_t)2 * n_slabs * chunks_kv + chunks_pos;
+    if (n_flags > kNoAllocMaxFlags)
+        return report_error(KVM_E_CAPACITY,
+                            "kv_compact_noalloc: 2 * n_slabs * ceil(moved / rows_per_chunk) + position chunks "
+                            "exceeds the 65536 read flags of the static scratch");
+
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return report_error(KVM_E_CUDA, "kv_compact_noalloc: no usable current device");
+    if (!g_noalloc_addr[dev]) {
+        void* addr = nullptr;
+        e = cudaGetSymbolAddress(&addr, kvm_noalloc_scratch);
+        if (e != cudaSuccess || !addr)
+            return report_error(KVM_E_CUDA, "kv_compact_noalloc: cudaGetSymbolAddress of the scratch failed");
+        g_noalloc_addr[dev] = static_cast<uint32_t*>(addr);
+    }
+    uint32_t* scratch = g_noalloc_addr[dev];
+    *new_live_out = L_new;
+    if (moved <= 0) return KVM_OK;
+
+    cudaStream_t s = (cudaStream_t)stream;
+    // tickets and the flags this call uses start at zero (the array keeps the
+    // previous call's contents); epoch 1 then marks "chunk read"
+    uint32_t* tickets = scratch + 64;
+    uint32_t* flags = tickets + kNoAllocTickets;
+    e = cudaMemsetAsync(tickets, 0, sizeof(uint32_t) * (2 * n_slabs + 1), s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(flags, 0, sizeof(uint32_t) * (size_t)n_flags, s);
+    if (e != cudaSuccess) return report_error(KVM_E_CUDA, "kv_compact_noalloc: clearing the scratch failed");
+
+    p.n_chars = 1;
+    p.n_kv_slabs = 2 * n_slabs;
+    p.vec_per_row = vec_per_row;
+    p.rows_kv = rows_kv;
+    p.rows_pos = rows_pos;
+    p.epoch = 1;
+    p.slab_rows = slab_rows;
+    p.K = static_cast<uint4*>(K);
+    p.V = static_cast<uint4*>(V);
+    p.pos = positions;
+    p.tickets = reinterpret_cast<int32_t*>(tickets);
+    p.flags = flags;
+    p.err = reinterpret_cast<int32_t*>(scratch);
+    CompactChar& c = p.ch[0];
+    c.L_new = L_new;
+    c.first = span_begin[0];
+    c.seg_off = 0;
+    c.n_seg = n_spans;
+    c.cap_off = 0;
+    c.chunks_kv = chunks_kv;
+    c.chunks_pos = chunks_pos;
+    c.blk_off = 0;
+    c.flag_off = 0;
+    p.total_blocks = p.n_kv_slabs * chunks_kv + chunks_pos;
+    launch_kv_compact(p, s);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return report_error(KVM_E_CUDA, "kv_compact_noalloc: kernel launch failed");
+    return KVM_OK;
+}

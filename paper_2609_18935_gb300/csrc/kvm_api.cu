@@ -815,3 +815,9 @@ extern "C" kvm_status kvm_profile_read(kvm_ctx* c, int32_t kernel, int64_t* laun
     }
     return KVM_OK;
 }
+
+namespace kvm {
+// Lets other translation units of the library report a failure through
+// kvm_last_error().
+kvm_status report_error(kvm_status code, const char* msg) { return fail(code, "%s", msg); }
+}  // namespace kvm

@@ -135,4 +135,7 @@ struct GdnParams {
 
 void launch_gdn_chunk_scan(const GdnParams& p, cudaStream_t s);
 
+// Set the text returned by kvm_last_error() and return `code`.
+int report_error(int code, const char* msg);
+
 }  // namespace kvm

@@ -74,6 +74,9 @@ _SIGS = {
     "kvm_check": (C.c_int, [C.c_void_p, C.c_void_p]),
     "kvm_launch_count": (C.c_int64, [C.c_void_p]),
     "kvm_fork": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "kvm_kv_compact_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int64, C.c_int32,
+                                         C.c_int32, C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32),
+                                         C.POINTER(C.c_int32), C.c_void_p]),
     "kvm_profile_enable": (C.c_int, [C.c_void_p, C.c_int32]),
     "kvm_profile_read": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double),
                                    C.c_int32]),
@@ -133,6 +136,22 @@ def _stream(stream) -> int:
     import torch
     s = stream if stream is not None else torch.cuda.current_stream()
     return s.cuda_stream
+
+
+def kv_compact_noalloc(K, V, positions, live, span_begin, span_end, stream=None) -> int:
+    """kvm_kv_compact_noalloc on caller-owned buffers (no allocation anywhere).
+
+    K, V: CUDA bf16 tensors [n_slabs][slab_rows][head_dim]; positions: CUDA
+    int32 [slab_rows] or None.  Returns the new live length."""
+    import torch
+    load_library()
+    n_slabs, rows, D = K.shape
+    sb, se = _i32(span_begin), _i32(span_end)
+    new_live = C.c_int32()
+    _check(_lib.kvm_kv_compact_noalloc(_dptr(K, torch.bfloat16), _dptr(V, torch.bfloat16),
+                                       _dptr(positions, torch.int32), n_slabs, rows, D, int(live), len(sb),
+                                       _p32(sb), _p32(se), C.byref(new_live), _stream(stream)))
+    return new_live.value
 
 
 class Context:
