@@ -18,6 +18,7 @@
 
 #include "../../include/kvm.h"
 #include "kvm_internal.cuh"
+#include "tma_host.h"
 
 using namespace kvm;
 
@@ -48,7 +49,7 @@ kvm_status fail(kvm_status code, const char* fmt, ...) {
         if (e_ != cudaSuccess) return fail(KVM_E_CUDA, "kernel launch failed: %s", cudaGetErrorString(e_)); \
     } while (0)
 
-constexpr int kItemCap = 1216;      // work items that keep a partial accumulator (8 per SM at 152 SMs)
+constexpr int kItemCap = 1024;      // attention work items that may keep a split partial
 
 }  // namespace
 
@@ -90,6 +91,7 @@ struct kvm_ctx {
     size_t stage_bytes[5] = {0, 0, 0, 0, 0};
     size_t stage_out_bytes = 0;
     double inv_freq[kMaxRotaryHalf] = {};
+    CUtensorMap tmap_q, tmap_k, tmap_v;   // TMA maps of q_rot, K, V (attention layers only)
     int64_t launches = 0;
     int rows_kv = 0, rows_pos = 0;
     // per-kernel timing (kvm_profile_*)
@@ -281,8 +283,8 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
     if (e == cudaSuccess) e = alloc_zero(&c->pos, c->n_attn ? (size_t)c->T_cap : 0);
     if (e == cudaSuccess) e = alloc_zero(&c->S, (size_t)c->n_gdn * n_chars * c->H * c->dv * c->dk);
     if (e == cudaSuccess) e = alloc_zero(&c->q_rot, c->n_attn ? (size_t)max_tail_tokens * c->Hq * c->D : 0);
-    if (e == cudaSuccess) e = alloc_zero(&c->part_o, c->n_attn ? (size_t)kItemCap * 64 * c->D : 0);
-    if (e == cudaSuccess) e = alloc_zero(&c->part_ml, c->n_attn ? (size_t)kItemCap * 64 * 2 : 0);
+    if (e == cudaSuccess) e = alloc_zero(&c->part_o, c->n_attn ? (size_t)kItemCap * kAttnRows * c->D : 0);
+    if (e == cudaSuccess) e = alloc_zero(&c->part_ml, c->n_attn ? (size_t)kItemCap * kAttnRows * 2 : 0);
     if (e == cudaSuccess) e = alloc_zero(&c->tickets, (size_t)n_chars * (n_kv_slabs + 1));
     if (e == cudaSuccess) e = alloc_zero(&c->flags, n_flags);
     if (e == cudaSuccess) e = alloc_zero(&c->err, 1);
@@ -300,6 +302,25 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         free_all(c);
         delete c;
         return fail(KVM_E_CUDA, "allocation failed: %s", cudaGetErrorString(e));
+    }
+    if (c->n_attn > 0) {
+        // TMA maps: rotated q as [max_tail][Hq][D] with a (64, g, 128/g) box;
+        // every layer's K and V as rows of D with a (64, 64) box
+        const uint64_t row_bytes = (uint64_t)c->D * 2;
+        const uint64_t qd[3] = {(uint64_t)c->D, (uint64_t)c->Hq, (uint64_t)max_tail_tokens};
+        const uint64_t qs[2] = {row_bytes, row_bytes * c->Hq};
+        const uint32_t qb[3] = {64, (uint32_t)c->g, (uint32_t)(kAttnRows / c->g)};
+        const uint64_t kd[2] = {(uint64_t)c->D, (uint64_t)c->n_attn * c->Hkv * c->T_cap};
+        const uint64_t ks[1] = {row_bytes};
+        const uint32_t kb[2] = {64, 64};
+        if (kd[1] > (uint64_t)INT32_MAX ||
+            !encode_bf16_sw128(&c->tmap_q, c->q_rot, 3, qd, qs, qb) ||
+            !encode_bf16_sw128(&c->tmap_k, c->K, 2, kd, ks, kb) ||
+            !encode_bf16_sw128(&c->tmap_v, c->V, 2, kd, ks, kb)) {
+            free_all(c);
+            delete c;
+            return fail(KVM_E_CUDA, "creating the TMA tensor maps failed");
+        }
     }
     *out = c;
     return KVM_OK;
@@ -557,9 +578,13 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
     thread_local static AttnParams p;
     std::memset(&p, 0, sizeof p);
     const int a = c->attn_idx[layer];
+    p.tmap_q = c->tmap_q;
+    p.tmap_k = c->tmap_k;
+    p.tmap_v = c->tmap_v;
+    p.attn_layer = a;
     p.n_chars = c->B;
     p.Hq = c->Hq; p.Hkv = c->Hkv; p.D = c->D; p.R = c->R; p.g = c->g;
-    p.tok_per_tile = 64 / c->g;
+    p.tok_per_tile = kAttnRows / c->g;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->D));
     p.slab_rows = c->T_cap;
     p.q = static_cast<const __nv_bfloat16*>(q);
@@ -585,9 +610,12 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
         ch.n_qtiles = (ch.M + p.tok_per_tile - 1) / p.tok_per_tile;
         tiles += c->Hkv * ch.n_qtiles;
     }
-    // key splits: fill about two waves of blocks when the tiles alone do not
+    // key splits: when the query tiles alone leave SMs idle, split each tile's
+    // keys so that the items fill one wave (1 block per SM at head_dim 256,
+    // 2 otherwise)
+    const int wave = c->num_sms * (c->D == 256 ? 1 : 2);
     int split = 1;
-    if (tiles < 2 * c->num_sms) split = std::min(16, (2 * c->num_sms + tiles - 1) / tiles);
+    if (tiles < wave) split = std::max(1, std::min(16, wave / tiles));
     while (split > 1 && (size_t)tiles * split > (size_t)kItemCap) --split;
     p.n_split = split;
     int items = 0;

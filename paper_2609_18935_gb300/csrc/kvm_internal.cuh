@@ -2,6 +2,7 @@
 // Everything here is private to libkvm; the public ABI is include/kvm.h.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -86,11 +87,17 @@ struct AttnChar {
 };
 
 struct AttnParams {
+    // TMA maps: rotated q [max_tail][Hq][D] (box 64 x g x 128/g), and every
+    // layer's K / V slabs as rows of D (box 64 x 64), 128-byte swizzle
+    CUtensorMap tmap_q;
+    CUtensorMap tmap_k;
+    CUtensorMap tmap_v;
+    int32_t attn_layer;   // index among attention layers
     int32_t n_chars;
     int32_t Hq, Hkv, D, R, g;
     int32_t n_split;      // key splits per query tile
     int32_t n_items;      // total work items
-    int32_t tok_per_tile; // tail tokens per 64-row query tile (64 / g)
+    int32_t tok_per_tile; // tail tokens per 128-row query tile (128 / g)
     float scale_log2;     // log2(e) / sqrt(D)
     int64_t slab_rows;    // rows per (layer, head) slab
     const __nv_bfloat16* q;       // caller's unrotated q  [sum M][Hq][D]
@@ -101,8 +108,8 @@ struct AttnParams {
     __nv_bfloat16* V;
     int32_t* pos;                 // [slab_rows]
     __nv_bfloat16* out;           // [sum M][Hq][D]
-    float* part_o;                // [n_items][64][D]
-    float* part_ml;               // [n_items][64][2]
+    float* part_o;                // [n_items][128][D]
+    float* part_ml;               // [n_items][128][2]
     int32_t* err;
     double inv_freq[kMaxRotaryHalf];
     AttnChar ch[kMaxChars];
@@ -111,6 +118,7 @@ struct AttnParams {
 void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s);
 void launch_tail_attention(const AttnParams& p, cudaStream_t s);
 void launch_attn_combine(const AttnParams& p, int n_tiles, cudaStream_t s);
+constexpr int kAttnRows = 128;   // query rows per attention tile
 
 // ----------------------------------------------------------------------------
 // gated delta rule

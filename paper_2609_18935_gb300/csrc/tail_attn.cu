@@ -1,25 +1,45 @@
-// True-tail prefill for one full-attention layer (Eq. 3, §4.2).
+// True-tail prefill for one full-attention layer (Eq. 3, §4.2): the kernels
+// around the tensor-core attention (tail_attn_tc.cu).
 //
-//  rope_append : rotate the tail's q and k at positions p + i (fp64 angle,
-//                fp32 rotation), append rotated k and v at live slots L' + i
-//                with their positions, and stage rotated q.
-//  tail_attention : causal GQA attention of the tail's queries over the
-//                compacted cache plus the tail itself.  A work item is
-//                (character, KV head, 64-row query tile, key split); the 64
-//                rows of a tile are (tail token, query head of the group)
-//                pairs, token-major, so one K/V tile serves all g heads of
-//                the group.  Online softmax in base 2; with one split the
-//                normalised output is written directly, otherwise the
-//                unnormalised partial accumulator and (max, sum) go to the
-//                workspace and attn_combine merges the splits.
+//  rope_append : rotate the tail's q and k at positions p + i, append the
+//                rotated k and v at live slots L' + i with their positions,
+//                and stage the rotated q for the attention's TMA loads.
+//                The angle pos * omega_d is formed and reduced modulo 2*pi in
+//                fp64 (positions far beyond the live length stay accurate),
+//                then sin/cos and the rotation run in fp32.
+//  attn_combine : merge the key splits of the attention: each split leaves
+//                an unnormalised accumulator and (reference max in log2
+//                units, sum); one warp per query row.
 #include "kvm_internal.cuh"
 
 namespace kvm {
 namespace {
 
-constexpr int kRows = 64;      // query rows per tile
-constexpr int kKeys = 64;      // keys per K/V tile
-constexpr int kThreads = 256;
+constexpr int kRows = kAttnRows;   // query rows per attention work item
+constexpr double kTwoPi = 6.283185307179586476925286766559;
+
+__device__ __forceinline__ float2 bf2_to_f2(uint32_t w) {
+    __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&w);
+    return __bfloat1622float2(h);
+}
+__device__ __forceinline__ uint32_t f2_to_bf2(float a, float b) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Rotate 8 pairs (lo[e], hi[e]) by the angles of dims d0 .. d0+7.
+__device__ __forceinline__ void rotate8(uint4& lo, uint4& hi, const float* cs, const float* sn, int d0) {
+    uint32_t* L = reinterpret_cast<uint32_t*>(&lo);
+    uint32_t* Hh = reinterpret_cast<uint32_t*>(&hi);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float2 x = bf2_to_f2(L[e]), y = bf2_to_f2(Hh[e]);
+        const int d = d0 + 2 * e;
+        const float c0 = cs[d], s0 = sn[d], c1 = cs[d + 1], s1 = sn[d + 1];
+        L[e] = f2_to_bf2(x.x * c0 - y.x * s0, x.y * c1 - y.y * s1);
+        Hh[e] = f2_to_bf2(y.x * c0 + x.x * s0, y.y * c1 + x.y * s1);
+    }
+}
 
 __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant__ AttnParams p) {
     const int n = blockIdx.x;                 // packed tail token
@@ -35,34 +55,65 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
     const int64_t pos = c.p + i;
     const int64_t slot = c.cap_off + c.L_prev + i;
     const int half = p.R / 2;
+    const int D = p.D;
 
     __shared__ float cs[kMaxRotaryHalf], sn[kMaxRotaryHalf];
     for (int d = threadIdx.x; d < half; d += blockDim.x) {
-        double sv, cv;
-        sincos((double)pos * p.inv_freq[d], &sv, &cv);
-        cs[d] = (float)cv;
-        sn[d] = (float)sv;
+        const double ang = (double)pos * p.inv_freq[d];
+        const double r = fma(-rint(ang * (1.0 / kTwoPi)), kTwoPi, ang);   // ang mod 2*pi, |r| <= pi
+        float sv, cv;
+        sincosf((float)r, &sv, &cv);
+        cs[d] = cv;
+        sn[d] = sv;
     }
     __syncthreads();
 
-    auto rotated = [&](const __nv_bfloat16* row, int d) -> float {
-        const float x = __bfloat162float(row[d]);
-        if (d >= p.R) return x;
-        if (d < half) return x * cs[d] - __bfloat162float(row[d + half]) * sn[d];
-        return x * cs[d - half] + __bfloat162float(row[d - half]) * sn[d - half];
-    };
-
-    for (int idx = threadIdx.x; idx < p.Hq * p.D; idx += blockDim.x) {
-        const int h = idx / p.D, d = idx % p.D;
-        const __nv_bfloat16* row = p.q + ((int64_t)n * p.Hq + h) * p.D;
-        p.q_rot[((int64_t)n * p.Hq + h) * p.D + d] = __float2bfloat16_rn(rotated(row, d));
-    }
-    for (int idx = threadIdx.x; idx < p.Hkv * p.D; idx += blockDim.x) {
-        const int h = idx / p.D, d = idx % p.D;
-        const __nv_bfloat16* krow = p.k_new + ((int64_t)n * p.Hkv + h) * p.D;
-        const int64_t dst = ((int64_t)h * p.slab_rows + slot) * p.D + d;
-        p.K[dst] = __float2bfloat16_rn(rotated(krow, d));
-        p.V[dst] = p.v_new[((int64_t)n * p.Hkv + h) * p.D + d];
+    const __nv_bfloat16* qrow = p.q + (int64_t)n * p.Hq * D;
+    __nv_bfloat16* qdst = p.q_rot + (int64_t)n * p.Hq * D;
+    const __nv_bfloat16* krow = p.k_new + (int64_t)n * p.Hkv * D;
+    const __nv_bfloat16* vrow = p.v_new + (int64_t)n * p.Hkv * D;
+    if ((half & 7) == 0) {
+        // 16-byte groups: group g < half/8 rotates with group g + half/8;
+        // groups from R/8 on are copied
+        const int rot = half / 8, copy = (D - p.R) / 8, per_head = rot + copy;
+        for (int idx = threadIdx.x; idx < (p.Hq + p.Hkv) * per_head; idx += blockDim.x) {
+            const int h = idx / per_head, gidx = idx % per_head;
+            const bool is_q = h < p.Hq;
+            const int hh = is_q ? h : h - p.Hq;
+            const __nv_bfloat16* src = is_q ? qrow + hh * D : krow + hh * D;
+            __nv_bfloat16* dst = is_q ? qdst + hh * D : p.K + ((int64_t)hh * p.slab_rows + slot) * D;
+            if (gidx < rot) {
+                const int d0 = gidx * 8;
+                uint4 a = *reinterpret_cast<const uint4*>(src + d0);
+                uint4 bb = *reinterpret_cast<const uint4*>(src + d0 + half);
+                rotate8(a, bb, cs, sn, d0);
+                *reinterpret_cast<uint4*>(dst + d0) = a;
+                *reinterpret_cast<uint4*>(dst + d0 + half) = bb;
+            } else {
+                const int d0 = p.R + (gidx - rot) * 8;
+                *reinterpret_cast<uint4*>(dst + d0) = *reinterpret_cast<const uint4*>(src + d0);
+            }
+        }
+        for (int idx = threadIdx.x; idx < p.Hkv * (D / 8); idx += blockDim.x) {
+            const int h = idx / (D / 8), d0 = (idx % (D / 8)) * 8;
+            *reinterpret_cast<uint4*>(p.V + ((int64_t)h * p.slab_rows + slot) * D + d0) =
+                *reinterpret_cast<const uint4*>(vrow + h * D + d0);
+        }
+    } else {
+        auto rotated = [&](const __nv_bfloat16* row, int d) -> float {
+            const float x = __bfloat162float(row[d]);
+            if (d >= p.R) return x;
+            if (d < half) return x * cs[d] - __bfloat162float(row[d + half]) * sn[d];
+            return x * cs[d - half] + __bfloat162float(row[d - half]) * sn[d - half];
+        };
+        for (int idx = threadIdx.x; idx < p.Hq * D; idx += blockDim.x)
+            qdst[idx] = __float2bfloat16_rn(rotated(qrow + (idx / D) * D, idx % D));
+        for (int idx = threadIdx.x; idx < p.Hkv * D; idx += blockDim.x) {
+            const int h = idx / D, d = idx % D;
+            const int64_t dst = ((int64_t)h * p.slab_rows + slot) * D + d;
+            p.K[dst] = __float2bfloat16_rn(rotated(krow + h * D, d));
+            p.V[dst] = vrow[h * D + d];
+        }
     }
     if (threadIdx.x == 0) p.pos[slot] = (int32_t)pos;
 }
@@ -83,207 +134,42 @@ __device__ __forceinline__ void decode_item(const AttnParams& p, int item, int& 
     kvh = local / p.ch[b].n_qtiles;
 }
 
-template <int D>
-__global__ void __launch_bounds__(kThreads) tail_attention_kernel(const __grid_constant__ AttnParams p) {
-    extern __shared__ float smem[];
-    float* Qs = smem;                                   // [64][D]   rotated q * log2(e)/sqrt(D)
-    float* Ss = Qs + kRows * D;                         // [64][65]  scores, then probabilities
-    __nv_bfloat16* Ks = reinterpret_cast<__nv_bfloat16*>(Ss + kRows * (kKeys + 1));  // [64][D+2]
-    __nv_bfloat16* Vs = Ks + kKeys * (D + 2);           // [64][D]
-    __shared__ float row_m[kRows], row_l[kRows], row_a[kRows];
-    __shared__ int row_lim[kRows];
-
-    const int tid = threadIdx.x;
-    const int item = blockIdx.x;
-    int b, kvh, qt, sp;
-    decode_item(p, item, b, kvh, qt, sp);
-    const AttnChar& c = p.ch[b];
-    const int g = p.g;
-    const int tok0 = qt * p.tok_per_tile;
-    const int tok_end = min(c.M, tok0 + p.tok_per_tile);
-    const int n_keys = c.L_prev + tok_end;              // keys any row of this tile may see
-    const int kt_total = (n_keys + kKeys - 1) / kKeys;
-    const int kt0 = (int)((int64_t)sp * kt_total / p.n_split);
-    const int kt1 = (int)((int64_t)(sp + 1) * kt_total / p.n_split);
-
-    // load the query tile (rows past the tail reuse the last token; never stored)
-    for (int idx = tid; idx < kRows * D; idx += kThreads) {
-        const int r = idx / D, d = idx % D;
-        const int tok = min(tok0 + r / g, c.M - 1);
-        const int hq = kvh * g + (r % g);
-        Qs[idx] = __bfloat162float(p.q_rot[((int64_t)(c.tail_off + tok) * p.Hq + hq) * D + d]) * p.scale_log2;
-    }
-    if (tid < kRows) {
-        const int tok = min(tok0 + tid / g, c.M - 1);
-        row_lim[tid] = c.L_prev + tok + 1;
-        row_m[tid] = -INFINITY;
-        row_l[tid] = 0.f;
-    }
-
-    const int ty = tid / 16, tx = tid % 16;
-    constexpr int DJ = D / 16;
-    float acc[4][DJ];
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < DJ; ++j) acc[i][j] = 0.f;
-
-    const __nv_bfloat16* Kbase = p.K + ((int64_t)kvh * p.slab_rows + c.cap_off) * D;
-    const __nv_bfloat16* Vbase = p.V + ((int64_t)kvh * p.slab_rows + c.cap_off) * D;
-
-    for (int kt = kt0; kt < kt1; ++kt) {
-        __syncthreads();
-        const int key0 = kt * kKeys;
-        for (int idx = tid; idx < kKeys * (D / 8); idx += kThreads) {
-            const int r = idx / (D / 8), d8 = (idx % (D / 8)) * 8;
-            uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
-            if (key0 + r < n_keys) {
-                kv = *reinterpret_cast<const uint4*>(Kbase + (int64_t)(key0 + r) * D + d8);
-                vv = *reinterpret_cast<const uint4*>(Vbase + (int64_t)(key0 + r) * D + d8);
-            }
-            const __nv_bfloat16* kh = reinterpret_cast<const __nv_bfloat16*>(&kv);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) Ks[r * (D + 2) + d8 + e] = kh[e];
-            *reinterpret_cast<uint4*>(Vs + r * D + d8) = vv;
-        }
-        __syncthreads();
-        // scores for rows ty*4+i, keys tx + 16*j
-        float s[4][4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-            for (int j = 0; j < 4; ++j) s[i][j] = 0.f;
-        for (int d = 0; d < D; ++d) {
-            float qv[4], kv[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) qv[i] = Qs[(ty * 4 + i) * D + d];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) kv[j] = __bfloat162float(Ks[(tx + 16 * j) * (D + 2) + d]);
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) s[i][j] = fmaf(qv[i], kv[j], s[i][j]);
-        }
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int r = ty * 4 + i, key = tx + 16 * j;
-                Ss[r * (kKeys + 1) + key] = (key0 + key < row_lim[r]) ? s[i][j] : -INFINITY;
-            }
-        __syncthreads();
-        // online softmax: 4 threads per row
-        {
-            const int r = tid / 4, q4 = tid % 4;
-            float mx = -INFINITY;
-#pragma unroll
-            for (int k = 0; k < 16; ++k) mx = fmaxf(mx, Ss[r * (kKeys + 1) + q4 + 4 * k]);
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-            const float m_old = row_m[r];
-            const float m_new = fmaxf(m_old, mx);
-            float sum = 0.f;
-#pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                float* sp_ = &Ss[r * (kKeys + 1) + q4 + 4 * k];
-                const float e = (m_new == -INFINITY) ? 0.f : exp2f(*sp_ - m_new);
-                *sp_ = e;
-                sum += e;
-            }
-            sum += __shfl_xor_sync(0xffffffffu, sum, 1);
-            sum += __shfl_xor_sync(0xffffffffu, sum, 2);
-            __syncwarp();
-            if (q4 == 0) {
-                const float a = (m_old == -INFINITY) ? 0.f : exp2f(m_old - m_new);
-                row_a[r] = a;
-                row_l[r] = row_l[r] * a + sum;
-                row_m[r] = m_new;
-            }
-        }
-        __syncthreads();
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float a = row_a[ty * 4 + i];
-#pragma unroll
-            for (int j = 0; j < DJ; ++j) acc[i][j] *= a;
-        }
-        for (int key = 0; key < kKeys; ++key) {
-            float pv[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) pv[i] = Ss[(ty * 4 + i) * (kKeys + 1) + key];
-#pragma unroll
-            for (int j = 0; j < DJ; ++j) {
-                const float vv = __bfloat162float(Vs[key * D + tx + 16 * j]);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) acc[i][j] = fmaf(pv[i], vv, acc[i][j]);
-            }
-        }
-    }
-    __syncthreads();
-
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int r = ty * 4 + i;
-        const int tok = tok0 + r / g;
-        if (tok >= c.M) continue;
-        const int hq = kvh * g + (r % g);
-        if (p.n_split == 1) {
-            const float inv = 1.f / row_l[r];
-            __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + hq) * D;
-#pragma unroll
-            for (int j = 0; j < DJ; ++j) o[tx + 16 * j] = __float2bfloat16_rn(acc[i][j] * inv);
-        } else {
-            float* o = p.part_o + ((int64_t)item * kRows + r) * D;
-#pragma unroll
-            for (int j = 0; j < DJ; ++j) o[tx + 16 * j] = acc[i][j];
-            if (tx == 0) {
-                p.part_ml[((int64_t)item * kRows + r) * 2 + 0] = row_m[r];
-                p.part_ml[((int64_t)item * kRows + r) * 2 + 1] = row_l[r];
-            }
-        }
-    }
-}
-
-// One block per (character, KV head, query tile): merge the key splits.
+// grid (tiles, kRows / 8): one warp per query row, lanes over head_dim.
 __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant__ AttnParams p) {
-    const int tile = blockIdx.x;             // item index / n_split
+    const int tile = blockIdx.x;
+    const int r = blockIdx.y * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
     int b, kvh, qt, sp;
     decode_item(p, tile * p.n_split, b, kvh, qt, sp);
     const AttnChar& c = p.ch[b];
-    const int item0 = tile * p.n_split;
+    const int tok = qt * p.tok_per_tile + r / p.g;
+    if (tok >= c.M) return;
     const int D = p.D;
-    for (int idx = threadIdx.x; idx < kRows * D; idx += blockDim.x) {
-        const int r = idx / D, d = idx % D;
-        const int tok = qt * p.tok_per_tile + r / p.g;
-        if (tok >= c.M) continue;
-        float mx = -INFINITY;
-        for (int s = 0; s < p.n_split; ++s)
-            mx = fmaxf(mx, p.part_ml[((int64_t)(item0 + s) * kRows + r) * 2]);
-        float num = 0.f, den = 0.f;
+    const int64_t item0 = (int64_t)tile * p.n_split;
+    float ms[16], ws[16];
+    float mx = -INFINITY;
+    for (int s = 0; s < p.n_split; ++s) {
+        ms[s] = p.part_ml[((item0 + s) * kRows + r) * 2];
+        mx = fmaxf(mx, ms[s]);
+    }
+    float den = 0.f;
+    for (int s = 0; s < p.n_split; ++s) {
+        ws[s] = (ms[s] == -INFINITY) ? 0.f : exp2f(ms[s] - mx);
+        den += ws[s] * p.part_ml[((item0 + s) * kRows + r) * 2 + 1];
+    }
+    const float inv = 1.f / den;
+    const int hq = kvh * p.g + (r % p.g);
+    __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + hq) * D;
+    for (int v4 = lane; v4 < D / 4; v4 += 32) {
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int s = 0; s < p.n_split; ++s) {
-            const float m = p.part_ml[((int64_t)(item0 + s) * kRows + r) * 2];
-            if (m == -INFINITY) continue;
-            const float w = exp2f(m - mx);
-            num += w * p.part_o[((int64_t)(item0 + s) * kRows + r) * D + d];
-            den += w * p.part_ml[((int64_t)(item0 + s) * kRows + r) * 2 + 1];
+            if (ws[s] == 0.f) continue;
+            const float4 x = *reinterpret_cast<const float4*>(p.part_o + ((item0 + s) * kRows + r) * D + v4 * 4);
+            acc.x += ws[s] * x.x; acc.y += ws[s] * x.y; acc.z += ws[s] * x.z; acc.w += ws[s] * x.w;
         }
-        const int hq = kvh * p.g + (r % p.g);
-        p.out[((int64_t)(c.tail_off + tok) * p.Hq + hq) * D + d] = __float2bfloat16_rn(num / den);
+        const uint2 packed = make_uint2(f2_to_bf2(acc.x * inv, acc.y * inv), f2_to_bf2(acc.z * inv, acc.w * inv));
+        *reinterpret_cast<uint2*>(o + v4 * 4) = packed;
     }
-}
-
-template <int D>
-void launch_attn_d(const AttnParams& p, cudaStream_t s) {
-    const size_t smem = sizeof(float) * (kRows * D + kRows * (kKeys + 1)) +
-                        sizeof(__nv_bfloat16) * (kKeys * (D + 2) + kKeys * D);
-    static unsigned long long configured = 0;   // one bit per device
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (!(configured >> (dev & 63) & 1ull)) {
-        cudaFuncSetAttribute(tail_attention_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        configured |= 1ull << (dev & 63);
-    }
-    tail_attention_kernel<D><<<p.n_items, kThreads, smem, s>>>(p);
 }
 
 }  // namespace
@@ -293,19 +179,9 @@ void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s) {
     rope_append_kernel<<<total_tokens, 128, 0, s>>>(p);
 }
 
-void launch_tail_attention(const AttnParams& p, cudaStream_t s) {
-    if (p.n_items <= 0) return;
-    switch (p.D) {
-        case 64: launch_attn_d<64>(p, s); break;
-        case 128: launch_attn_d<128>(p, s); break;
-        case 256: launch_attn_d<256>(p, s); break;
-        default: break;   // rejected on the host
-    }
-}
-
 void launch_attn_combine(const AttnParams& p, int n_tiles, cudaStream_t s) {
     if (n_tiles <= 0 || p.n_split <= 1) return;
-    attn_combine_kernel<<<n_tiles, 256, 0, s>>>(p);
+    attn_combine_kernel<<<dim3(n_tiles, kRows / 8), 256, 0, s>>>(p);
 }
 
 }  // namespace kvm
