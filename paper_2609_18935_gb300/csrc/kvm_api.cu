@@ -655,6 +655,7 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
     std::memset(&p, 0, sizeof p);
     p.n_chars = c->B;
     p.H = c->H; p.dk = c->dk; p.dv = c->dv;
+    p.dv_slice = c->dv / ((c->dv + 127) / 128);
     p.q = static_cast<const __nv_bfloat16*>(q);
     p.k = static_cast<const __nv_bfloat16*>(k);
     p.v = static_cast<const __nv_bfloat16*>(v);

@@ -130,6 +130,7 @@ struct GdnChar {
 
 struct GdnParams {
     int32_t n_chars, H, dk, dv;
+    int32_t dv_slice;         // rows of S per block (a multiple of 16, <= 128, dividing dv)
     const __nv_bfloat16* q;   // [sum M][H][dk]
     const __nv_bfloat16* k;
     const __nv_bfloat16* v;   // [sum M][H][dv]
