@@ -64,6 +64,20 @@ def gdn_flops(shape, tails):
     return 6.0 * shape.d_k * shape.d_v * shape.n_gdn_heads * sum(tails)
 
 
+def gdn_bytes(shape, tails):
+    """q, k, v, o (bf16) and alpha, beta (fp32) of every tail token and head,
+    plus the state read and written once per character and head."""
+    H, dk, dv = shape.n_gdn_heads, shape.d_k, shape.d_v
+    per_tok = H * ((2 * dk + 2 * dv) * 2 + 8)
+    return float(sum(tails) * per_tok + sum(1 for m in tails if m > 0) * H * dv * dk * 4 * 2)
+
+
+def rope_bytes(shape, tails):
+    """Read q, k, v of the tail; write the rotated q (staging), k and v."""
+    Hq, Hkv, D = shape.n_q_heads, shape.n_kv_heads, shape.head_dim
+    return float(sum(tails) * (Hq + 2 * Hkv) * D * 2 * 2)
+
+
 def compaction_bytes(shape, moved_rows):
     n_attn = len(shape.attn_layers)
     row = shape.n_kv_heads * shape.head_dim * 2 * 2 * n_attn + 4     # K and V of every layer + position
@@ -291,6 +305,8 @@ def run_kvm(args):
         rd["attn_flops"] = attention_flops(s, Lp, tails)        # per attention layer
         rd["gdn_flops"] = gdn_flops(s, tails)                   # per delta-rule layer
         rd["compact_bytes"] = compaction_bytes(s, moved)
+        rd["gdn_bytes"] = gdn_bytes(s, tails)                   # per delta-rule layer
+        rd["rope_bytes"] = rope_bytes(s, tails)                 # per attention layer
         rd["h2d"] = sum(t.numel() * t.element_size() for x in rd["h_in"].values() for t in x.values())
         rd["d2h"] = sum(t.numel() * t.element_size() for t in rd["h_out"].values())
 
@@ -358,15 +374,45 @@ def run_kvm(args):
     value = world * toks_rank / (total_ms / 1e3)
     e2e_value = world * sum(sum(rounds[r]["tails"]) for r in e2e_rids) / (e2e_ms / 1e3)
     hbm, tc_burst, tc_sust, peak_src = load_peaks()
-    n_attn = len(s.attn_layers)
-    attn = kernels.get("tail_attention", {"launches": 0, "total_ms": 0.0})
-    attn_flops_total = sum(rounds[r]["attn_flops"] * n_attn for r in rids)
-    achieved = attn_flops_total / (attn["total_ms"] / 1e3) / 1e12 if attn["total_ms"] > 0 else None
-    traffic = ncu_traffic("tail_attn.cu", "tail_attention")
-    roofline = {"bound": "tensor", "kernel": "tail_attention", "achieved": achieved, "peak": tc_burst,
-                "unit": "TFLOP/s", "frac": (achieved / tc_burst) if achieved else None,
-                "peak_kind": f"bf16 dense burst, {peak_src}", "traffic": traffic,
-                "algorithmic_flops_per_launch": attn_flops_total / max(1, attn["launches"])}
+    n_attn, n_gdn = len(s.attn_layers), len(s.gdn_layers)
+    # algorithmic work of every kernel family over the timed steps
+    work = {
+        "tail_attention": ("tensor", sum(rounds[r]["attn_flops"] * n_attn for r in rids)),
+        "gdn": ("hbm", sum(rounds[r]["gdn_bytes"] * n_gdn for r in rids)),
+        "kv_compact": ("hbm", sum(rounds[r]["compact_bytes"] for r in rids)),
+        "rope_append": ("hbm", sum(rounds[r]["rope_bytes"] * n_attn for r in rids)),
+    }
+    fam = {k: dict(v) for k, v in kernels.items()}
+    if "gdn_chunk_scan" in fam:
+        prep = fam.get("gdn_chunk_prep", {"total_ms": 0.0})
+        fam["gdn"] = {"launches": fam["gdn_chunk_scan"]["launches"],
+                      "total_ms": fam["gdn_chunk_scan"]["total_ms"] + prep["total_ms"]}
+    rooflines = {}
+    for name, (bound, amount) in work.items():
+        d = fam.get(name)
+        if not d or d["total_ms"] <= 0 or d["launches"] == 0:
+            continue
+        secs = d["total_ms"] / 1e3
+        if bound == "tensor":
+            ach, peak, unit = amount / secs / 1e12, tc_burst, "TFLOP/s"
+        else:
+            ach, peak, unit = amount / secs / 1e9, hbm, "GB/s"
+        rooflines[name] = {"bound": bound, "achieved": ach, "peak": peak, "unit": unit, "frac": ach / peak,
+                           "share": d["total_ms"] / total_ms, "per_launch": amount / d["launches"],
+                           "per_launch_unit": "flop" if bound == "tensor" else "byte"}
+    # the dominant kernel family is the one with the largest share of the step
+    dominant = max(rooflines, key=lambda k: rooflines[k]["share"]) if rooflines else None
+    kfile = {"tail_attention": "tail_attn_tc.cu", "gdn": "gdn_scan_tc.cu", "kv_compact": "kv_compact.cu",
+             "rope_append": "tail_attn.cu"}
+    roofline = None
+    if dominant:
+        rf = rooflines[dominant]
+        roofline = {"bound": rf["bound"], "kernel": dominant, "achieved": rf["achieved"], "peak": rf["peak"],
+                    "unit": rf["unit"], "frac": rf["frac"],
+                    "peak_kind": (f"bf16 dense burst, {peak_src}" if rf["bound"] == "tensor"
+                                  else f"HBM copy bandwidth, {peak_src}"),
+                    "traffic": ncu_traffic(kfile[dominant], dominant),
+                    "algorithmic_per_launch": rf["per_launch"], "share_of_step": rf["share"]}
     if rank != 0:
         return
     # ---- CPU oracle sample (rank 0 only, single GPU runs only)
@@ -381,16 +427,6 @@ def run_kvm(args):
     for name, d in kernels.items():
         per_kernel[name] = {"launches": d["launches"], "avg_us": 1e3 * d["total_ms"] / d["launches"],
                             "share": d["total_ms"] / total_ms}
-    gdn = kernels.get("gdn_chunk_scan")
-    comp = kernels.get("kv_compact")
-    extra = {}
-    if gdn:
-        gf = sum(rounds[r]["gdn_flops"] * len(s.gdn_layers) for r in rids)
-        extra["gdn_chunk_scan_tflops"] = gf / (gdn["total_ms"] / 1e3) / 1e12
-    if comp:
-        cb = sum(rounds[r]["compact_bytes"] for r in rids)
-        extra["kv_compact_gbs"] = cb / (comp["total_ms"] / 1e3) / 1e9
-        extra["kv_compact_hbm_frac"] = extra["kv_compact_gbs"] / hbm
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
@@ -407,7 +443,7 @@ def run_kvm(args):
                 "ms_per_step": e2e_ms / args.steps},
         "gpu_launches": launches,
         "kernels": per_kernel,
-        "derived": extra,
+        "rooflines": rooflines,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

@@ -68,7 +68,7 @@ typedef struct kvm_ctx kvm_ctx;
  * Delta-rule layers: n_gdn_heads heads with key dim d_k and value dim d_v.
  * Supported: D in {64, 128, 256}; rotary_dim even, <= D; group size
  * n_q_heads/n_kv_heads a power of two <= 64; d_k in {64, 128}; d_v a
- * multiple of 32, <= 256. */
+ * multiple of 32, <= 128. */
 typedef struct kvm_model_desc {
     int32_t n_layers;
     const int32_t* layer_kind;     /* host [n_layers] */
@@ -262,7 +262,7 @@ kvm_status kvm_fork(kvm_ctx* dst, const kvm_ctx* src, void* stream);
  * Events come from a pool made at enable time (4096 launches between
  * reads); launches beyond it are counted but not timed. */
 enum { KVM_K_COMPACT = 0, KVM_K_ROPE_APPEND = 1, KVM_K_ATTENTION = 2, KVM_K_ATTN_COMBINE = 3,
-       KVM_K_GDN = 4, KVM_K_GATHER = 5, KVM_K_COUNT = 6 };
+       KVM_K_GDN = 4, KVM_K_GATHER = 5, KVM_K_GDN_PREP = 6, KVM_K_COUNT = 7 };
 kvm_status kvm_profile_enable(kvm_ctx* ctx, int32_t enable);
 kvm_status kvm_profile_read(kvm_ctx* ctx, int32_t kernel, int64_t* launches, double* total_ms,
                             int32_t reset);

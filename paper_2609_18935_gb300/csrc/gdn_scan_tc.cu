@@ -2,26 +2,29 @@
 // (Eq. 3 for a recurrent layer; Gated DeltaNet, the layer family of §4.1):
 //     S_t = alpha_t S_{t-1} (I - beta_t k_t k_t^T) + beta_t v_t k_t^T,  o_t = S_t q_t.
 //
-// One block per (character, head, slice of d_v rows of S); 256 threads.  Warp
-// w reads TMEM lanes 32*(w % 4) .. +31, so TMEM row r is shared by one thread
-// of warp w and one of warp w + 4, which split its columns.  The state slice
-// lives in TMEM as S^T (lanes = d_k index c, columns = d_v index r, fp32).
-// Chunks of C = 64 tokens are processed in order.  With g_t = sum_{u<=t}
-// log alpha_u, G_t = exp(g_t) and w_j = beta_j exp(g_C - g_j):
-//   KK, QK   = [K;Q] K^T                                  (MMA)
+// Chunks of C = 64 tail tokens.  With g_t = sum_{u<=t} log alpha_u (within the
+// chunk), G_t = exp(g_t) and w_j = beta_j exp(g_C - g_j):
+//   KK, QK   = [K;Q] K^T
 //   L        = strict_lower(exp(g_t - g_j) beta_j KK),  A = lower(exp(g_t - g_j) beta_j QK)
-//   X        = [I; A] (I + L)^-1 = [T; A T]                (per-row triangular solve, fp32)
-//   W  = X G K,  U = X V  (rows 0..63: W, U; rows 64..127: A W, A U)       (MMA)
+//   X        = [I; A] (I + L)^-1 = [T; A T]
+//   W  = T G K,  U = T V,  A W,  A U                    (= X G K and X V)
 //   Q' = G Q - A W
-//   [W S0^T; Q' S0^T] = [W; Q'] S0^T                      (MMA with the state)
-//   E  = U - W S0^T,   O = A U + Q' S0^T  (= G Q S0^T + A E)
-//   S^T = G_C S0^T + K^T diag(w) E                          (MMA, accumulated in TMEM)
-// Tensor-core operands are bf16.  The inputs K, Q, V are exact in bf16 and
-// are used in place (K and V as MN-major operands in their natural row
-// layout).  Every computed fp32 operand x (X, W, Q', S, w E) is split into
-// x_hi = bf16(x) and x_lo = bf16(x - x_hi); a product of two split operands
-// is hi*hi + hi*lo + lo*hi with fp32 accumulation, about 2^-15 relative
-// accuracy.  The master state stays fp32 in TMEM.
+//   E  = U - W S0^T,   O = A U + Q' S0^T               (= G Q S0^T + A E)
+//   S^T = G_C S0^T + K^T diag(w) E
+// Everything above the line "E = ..." is independent of the state, so it runs
+// in a prep kernel with one block per (chunk, head), all chunks in parallel;
+// it leaves per (chunk, head) a record with [W; Q'] and K as ready-made MMA
+// operand images, U and A U in fp32, w and G_C.  The scan kernel then walks
+// the chunks of each (character, head, d_v slice) in order with the state in
+// TMEM: one bulk copy of the next record's images (double-buffered), the MMA
+// [W; Q'] S0^T, E and O, and the state update.
+//
+// Tensor-core operands are bf16.  K, Q, V are exact in bf16 and used in place
+// (K and V as MN-major operands in their natural row layout).  Every computed
+// fp32 operand x (X, W, Q', S, w E) is split into x_hi = bf16(x) and
+// x_lo = bf16(x - x_hi); a product with a split operand is hi*hi + hi*lo +
+// lo*hi (or hi + lo against an exact operand) with fp32 accumulation, about
+// 2^-15 relative accuracy.  The master state stays fp32 in TMEM.
 #include "kvm_internal.cuh"
 #include "sm100_ptx.cuh"
 
@@ -32,30 +35,26 @@ using namespace ptx;
 
 constexpr int C = 64;            // chunk length
 constexpr int kThreads = 256;
-constexpr int DVMAX = 128;       // d_v rows per block
+constexpr int DVMAX = 128;       // d_v rows per scan block
+constexpr int DVP = 256;         // largest d_v the prep kernel stages
 constexpr int LSTRIDE = 68;      // fp32 row stride of the L scratch (conflict-free row vectors)
 
+// Workspace record of one (chunk, head):
+//   [W;Q'] hi | [W;Q'] lo   (128 x DK bf16 each, K-major 128-byte-swizzled image)
+//   K                       (64 x DK bf16, 128-byte-swizzled image, rows = tokens)
+//   U | A U                 (fp32 [128][dv], rows 0..63 U, 64..127 A U; the
+//                            16-byte chunk c of row r is stored at chunk
+//                            (c + r) mod (dv/4), so row-parallel reads of a
+//                            copy in shared memory do not collide on banks)
+//   w[64], G_C              (fp32)
 template <int DK>
-struct GCfg {
-    // byte offsets of the shared-memory regions (each 1024-aligned)
-    static constexpr int KQ = 128 * DK * 2;                  // [K;Q] bf16, K-major, 128 rows
-    static constexpr int V = C * DVMAX * 2;                  // V bf16, rows j (MN-major operand)
-    static constexpr int TILE128 = 128 * 64 * 2;             // 128 x 64 bf16 K-major tile (16 KB)
-    static constexpr int WQ = 2 * 128 * DK * 2;              // [W;Q'] hi, lo
-    static constexpr int RA = (WQ > 32768 + 2 * TILE128) ? WQ : 32768 + 2 * TILE128;   // L + X*G hi/lo, then [W;Q']
-    static constexpr int RX = 2 * TILE128;                   // X hi, lo
-    static constexpr int RS = 2 * DK * DVMAX * 2;            // S hi, lo (rows c); w E hi, lo aliased
-    static constexpr int OFF_KQ = 0;
-    static constexpr int OFF_V = OFF_KQ + KQ;
-    static constexpr int OFF_A = OFF_V + V;
-    static constexpr int OFF_X = OFF_A + RA;
-    static constexpr int OFF_S = OFF_X + RX;
-    static constexpr int OFF_BAR = OFF_S + RS;
-    static constexpr int SMEM = OFF_BAR + 64 + 1024;
-    // TMEM columns
-    static constexpr uint32_t T_D = 0;          // KK/QK (64 cols), later [W;Q'] S0^T (dv cols)
-    static constexpr uint32_t T_WU = 128;       // [W | U] (DK + dv cols)
-    static constexpr uint32_t T_S = 384;        // S^T     (dv cols)
+struct Rec {
+    static constexpr int64_t WQH = 128 * DK * 2;
+    static constexpr int64_t KIMG = 64 * DK * 2;
+    static constexpr int64_t IMG = 2 * WQH + KIMG;
+    static __host__ __device__ int64_t uau_off() { return IMG; }
+    static __host__ __device__ int64_t misc_off(int dv) { return IMG + (int64_t)128 * dv * 4; }
+    static __host__ __device__ int64_t bytes(int dv) { return IMG + (int64_t)128 * dv * 4 + 512; }
 };
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
@@ -77,44 +76,65 @@ __device__ __forceinline__ void split8(const float* x, uint4& hi, uint4& lo) {
     lo = make_uint4(lw[0], lw[1], lw[2], lw[3]);
 }
 
+__device__ __forceinline__ int find_char_by_chunk(const GdnParams& p, int chunk) {
+    int lo = 0, hi = p.n_chars - 1;              // last b with chunk_off <= chunk
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.ch[mid].chunk_off <= chunk) lo = mid; else hi = mid - 1;
+    }
+    return lo;
+}
+
+// ============================================================================
+// prep: one block per (chunk, head)
+// ============================================================================
 template <int DK>
-__global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_constant__ GdnParams p) {
-    using G = GCfg<DK>;
+struct PrepCfg {
+    static constexpr int KQ = 128 * DK * 2;                  // [K;Q] bf16, K-major, 128 rows
+    static constexpr int V = C * DVP * 2;                    // V bf16, rows j (MN-major operand)
+    static constexpr int TILE128 = 128 * 64 * 2;             // 128 x 64 bf16 K-major tile
+    static constexpr int OFF_KQ = 0;
+    static constexpr int OFF_V = OFF_KQ + KQ;
+    static constexpr int OFF_L = OFF_V + V;                  // fp32 [64][LSTRIDE] L, then the A rows
+    static constexpr int OFF_XG = OFF_L + 36864;             // X G hi, lo
+    static constexpr int OFF_X = OFF_XG + 2 * TILE128;       // X hi, lo
+    static constexpr int OFF_BAR = OFF_X + 2 * TILE128;
+    static constexpr int SMEM = OFF_BAR + 64 + 1024;
+    static constexpr uint32_t T_D = 0;                       // KK / QK (64 cols)
+    static constexpr uint32_t T_WU = 128;                    // [W | U] (DK + dv cols)
+};
+
+template <int DK>
+__global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_constant__ GdnParams p) {
+    using G = PrepCfg<DK>;
+    using R = Rec<DK>;
     extern __shared__ uint8_t smem_raw[];
-    // 1024-byte alignment by pointer arithmetic on the shared array, so that the
-    // accesses below stay shared-memory accesses
     uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const uint32_t sb = smem_u32(smem);
     auto V4 = [&](uint32_t off) -> uint4& { return *reinterpret_cast<uint4*>(smem + off); };
-    constexpr uint32_t oKQ = G::OFF_KQ, oV = G::OFF_V, oA = G::OFF_A, oX = G::OFF_X, oS = G::OFF_S;
-    constexpr uint32_t oL = oA;                                  // fp32 [64][LSTRIDE]
-    constexpr uint32_t oXG = oA + 32768;                         // X G hi, lo (K-major 128 x 64)
+    constexpr uint32_t oKQ = G::OFF_KQ, oV = G::OFF_V, oXG = G::OFF_XG, oX = G::OFF_X;
     constexpr uint32_t T128 = G::TILE128;
-    constexpr uint32_t WQH = 128 * DK * 2;                       // one [W;Q'] half
-    constexpr uint32_t SH = DK * DVMAX * 2;                      // one S half
-    constexpr uint32_t WEH = C * DVMAX * 2;                      // one w E half
-    float* Lm = reinterpret_cast<float*>(smem + oL);
+    float* Lm = reinterpret_cast<float*>(smem + G::OFF_L);
     uint64_t* bar = reinterpret_cast<uint64_t*>(smem + G::OFF_BAR);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + G::OFF_BAR + 8);
     const uint32_t mbar = smem_u32(bar);
-    __shared__ float gs[C], bs[C], Gs[C], ws[C];
+    float* Bm = Lm + 64 * LSTRIDE;                   // fp32 [64][LSTRIDE]: rows of A (right-hand sides)
+    __shared__ float gs[C], bs[C], Gs[C], g2[C];
     __shared__ volatile int abort_flag;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int q4 = warp & 3, hf = warp >> 2;
-    const int row = q4 * 32 + lane;                  // TMEM lane owned (with its twin in warp w ^ 4)
+    const int row = q4 * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
-    const int dvs = p.dv_slice;
-    const int r0 = blockIdx.x * dvs;
-    const int h = blockIdx.y;
-    const int b = blockIdx.z;
-    const GdnChar ch = p.ch[b];
-    if (ch.M <= 0) return;                           // uniform per block
     const int H = p.H, dv = p.dv;
-    float* Sg = p.S + ((int64_t)b * H + h) * dv * DK;
-    // columns of a dv-wide TMEM row handled by this thread: [dlo, dhi)
-    const int dhalf = ((dvs / 2) + 31) / 32 * 32;
-    const int dlo = hf * dhalf, dhi = min(dvs, dlo + dhalf);
+    const int chunk = blockIdx.x / H, h = blockIdx.x % H;
+    const int b = find_char_by_chunk(p, chunk);
+    const GdnChar ch = p.ch[b];
+    const int c0 = (chunk - ch.chunk_off) * C;
+    if (c0 >= ch.M) return;                          // uniform per block (not reached for valid grids)
+    const int n = min(C, ch.M - c0);
+    const int64_t tok0 = ch.tail_off + c0;
+    uint8_t* rec = p.work + ((int64_t)chunk * H + h) * p.rec_bytes;
 
     if (tid == 0) {
         abort_flag = 0;
@@ -125,12 +145,319 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
         tmem_alloc(smem_u32(tmem_slot), 512);
         tmem_relinquish();
     }
+    // ---- loads (every global load issued before the shared stores)
+    {
+        constexpr int NKQ = 128 * (DK / 8) / kThreads;
+        constexpr int NV = C * (DVP / 8) / kThreads;
+        uint4 kq[NKQ], vv[NV];
+#pragma unroll
+        for (int u = 0; u < NKQ; ++u) {
+            const int i = tid + u * kThreads;
+            const int rr = i / (DK / 8), c8 = (i % (DK / 8)) * 8, t = rr & 63;
+            kq[u] = t < n ? __ldg(reinterpret_cast<const uint4*>((rr < 64 ? p.k : p.q) + ((tok0 + t) * H + h) * DK + c8))
+                          : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+            const int i = tid + u * kThreads;
+            const int t = i / (dv / 8), r8 = (i % (dv / 8)) * 8;
+            vv[u] = (i < C * (dv / 8) && t < n) ? __ldg(reinterpret_cast<const uint4*>(p.v + ((tok0 + t) * H + h) * dv + r8))
+                                                : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int u = 0; u < NKQ; ++u) {
+            const int i = tid + u * kThreads;
+            const int rr = i / (DK / 8), c8 = (i % (DK / 8)) * 8;
+            V4(oKQ + sw128_off16(rr, c8, 128)) = kq[u];
+            // the K image of the record (rows = tokens, 64-row regions)
+            if (rr < 64) *reinterpret_cast<uint4*>(rec + 2 * R::WQH + sw128_off16(rr, c8, 64)) = kq[u];
+        }
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+            const int i = tid + u * kThreads;
+            if (i < C * (dv / 8)) V4(oV + sw128_off16(i / (dv / 8), (i % (dv / 8)) * 8, C)) = vv[u];
+        }
+    }
+    if (tid < 32) {
+        float x0 = tid < n ? logf(__ldg(p.alpha + (tok0 + tid) * H + h)) : 0.f;
+        float x1 = tid + 32 < n ? logf(__ldg(p.alpha + (tok0 + tid + 32) * H + h)) : 0.f;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const float y0 = __shfl_up_sync(0xffffffffu, x0, o);
+            const float y1 = __shfl_up_sync(0xffffffffu, x1, o);
+            if (tid >= o) { x0 += y0; x1 += y1; }
+        }
+        x1 += __shfl_sync(0xffffffffu, x0, 31);
+        gs[tid] = x0;
+        gs[tid + 32] = x1;
+        bs[tid] = tid < n ? __ldg(p.beta + (tok0 + tid) * H + h) : 0.f;
+        bs[tid + 32] = tid + 32 < n ? __ldg(p.beta + (tok0 + tid + 32) * H + h) : 0.f;
+    }
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    if (tid < C) {
+        Gs[tid] = expf(gs[tid]);
+        g2[tid] = gs[tid] * 1.4426950408889634f;          // log2 domain for the decays
+        float* misc = reinterpret_cast<float*>(rec + R::misc_off(dv));
+        misc[tid] = tid < n ? bs[tid] * expf(gs[n - 1] - gs[tid]) : 0.f;     // w_j
+        if (tid == 0) misc[C] = expf(gs[n - 1]);                            // G_C
+    }
+    uint32_t phase = 0;
+    bool ok = true;
+    auto mma_wait = [&]() -> bool {
+        bool r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait);
+        phase ^= 1;
+        r = __syncthreads_and(r);
+        tc_fence_after();
+        return r;
+    };
+    const uint32_t kq_region = 128 * 128;
+    // ---------------------------------------------------------------- KK, QK
+    if (tid == 0) {
+#pragma unroll
+        for (int ks = 0; ks < DK / 16; ++ks) {
+            const uint32_t off = (ks >> 2) * kq_region + (ks & 3) * 32;
+            mma_bf16(tmem + G::T_D, smem_desc_sw128(sb + oKQ + off, 16, 1024), smem_desc_sw128(sb + oKQ + off, 16, 1024),
+                     idesc_bf16_f32(128, C, false), ks > 0);
+        }
+        mma_commit(mbar);
+    }
+    ok = mma_wait();                                // also publishes Gs
+    // ---------------------------------------------------------------- L (rows < 64), A (rows >= 64)
+    if (ok) {
+        // thread (row, hf) handles columns hf*32 .. hf*32+31 of TMEM row `row`
+        uint32_t v[32];
+        tmem_ld32(tmem + lane_off + G::T_D + hf * 32, v);
+        tmem_ld_wait();
+        const int t = row & 63;
+        const float gt2 = g2[t];
+        float* dst = (row < 64 ? Lm : Bm) + t * LSTRIDE + hf * 32;
+#pragma unroll
+        for (int j4 = 0; j4 < 32; j4 += 4) {
+            float y[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int j = hf * 32 + j4 + e;
+                const bool keep = (row < 64) ? (j < t) : (j <= t);
+                y[e] = (keep && t < n) ? ex2(gt2 - g2[j]) * bs[j] * __uint_as_float(v[j4 + e]) : 0.f;
+            }
+            *reinterpret_cast<float4*>(dst + j4) = make_float4(y[0], y[1], y[2], y[3]);
+        }
+    }
+    __syncthreads();
+    // ---------------------------------------------------------------- X = [I; A] (I + L)^-1
+    // Two threads of one warp per row p (tid = 2p + h2): thread h2 owns the
+    // 8-column groups j8 = 16k + 8*h2; x (I + L) = b is solved right-looking,
+    // x_j -= x_i L[i][j] for j < i, i from 63 down, with x_i passed by shuffle.
+    if (ok) {
+        const int pr = tid >> 1, h2 = tid & 1;
+        float xs[32];                                 // xs[8k + e] = x[16k + 8 h2 + e]
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int j8 = 16 * k + 8 * h2;
+            if (pr < 64) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) xs[8 * k + e] = (j8 + e == pr) ? 1.f : 0.f;
+            } else {
+                const float4 b0 = *reinterpret_cast<const float4*>(Bm + (pr - 64) * LSTRIDE + j8);
+                const float4 b1 = *reinterpret_cast<const float4*>(Bm + (pr - 64) * LSTRIDE + j8 + 4);
+                xs[8 * k + 0] = b0.x; xs[8 * k + 1] = b0.y; xs[8 * k + 2] = b0.z; xs[8 * k + 3] = b0.w;
+                xs[8 * k + 4] = b1.x; xs[8 * k + 5] = b1.y; xs[8 * k + 6] = b1.z; xs[8 * k + 7] = b1.w;
+            }
+        }
+#pragma unroll
+        for (int i = C - 1; i > 0; --i) {
+            const int owner = (i >> 3) & 1;
+            const float xi = __shfl_sync(0xffffffffu, xs[8 * (i >> 4) + (i & 7)], (lane & ~1) | owner);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int j8 = 16 * k + 8 * h2;
+                if (j8 < i) {
+                    const float4 l0 = *reinterpret_cast<const float4*>(Lm + i * LSTRIDE + j8);
+                    const float4 l1 = *reinterpret_cast<const float4*>(Lm + i * LSTRIDE + j8 + 4);
+                    const float lv[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) xs[8 * k + e] = fmaf(-xi, lv[e], xs[8 * k + e]);   // L[i][j] = 0 for j >= i
+                }
+            }
+        }
+        // operands: X G (for W) and X (for U), K-major rows
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int j8 = 16 * k + 8 * h2;
+            float xg[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) xg[e] = xs[8 * k + e] * Gs[j8 + e];
+            uint4 hi, lo;
+            split8(xg, hi, lo);
+            const uint32_t off = sw128_off16(pr, j8, 128);
+            V4(oXG + off) = hi;
+            V4(oXG + T128 + off) = lo;
+            split8(xs + 8 * k, hi, lo);
+            V4(oX + off) = hi;
+            V4(oX + T128 + off) = lo;
+        }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    // ---------------------------------------------------------------- [W | U] = X [G K | V]
+    if (ok && tid == 0) {
+        tc_fence_after();
+#pragma unroll
+        for (int ks = 0; ks < C / 16; ++ks) {
+            const uint64_t bk = smem_desc_sw128(sb + oKQ + ks * 2048, kq_region, 1024);
+            const uint64_t bvv = smem_desc_sw128(sb + oV + ks * 2048, C * 128, 1024);
+#pragma unroll
+            for (int part = 0; part < 2; ++part) {
+                const uint32_t ao = part * T128 + ks * 32;
+                mma_bf16(tmem + G::T_WU, smem_desc_sw128(sb + oXG + ao, 16, 1024), bk,
+                         idesc_bf16_f32(128, DK, true), (ks | part) != 0);
+                mma_bf16(tmem + G::T_WU + DK, smem_desc_sw128(sb + oX + ao, 16, 1024), bvv,
+                         idesc_bf16_f32(128, dv, true), (ks | part) != 0);
+            }
+        }
+        mma_commit(mbar);
+    }
+    if (ok) ok = mma_wait();
+    // ---------------------------------------------------------------- record: [W; Q'] image, U | A U
+    if (ok) {
+        const int t = row & 63;
+        const float gt = Gs[t];
+        for (int cb = hf * (DK / 2); cb < (hf + 1) * (DK / 2); cb += 32) {
+            uint32_t v[32];
+            tmem_ld32(tmem + lane_off + G::T_WU + cb, v);
+            tmem_ld_wait();
+            float y[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) y[j] = __uint_as_float(v[j]);
+            if (row >= 64) {
+                // Q' = G Q - A W ; row `row` of [K;Q] holds q_t
+#pragma unroll
+                for (int j8 = 0; j8 < 32; j8 += 8) {
+                    const uint4 q8 = V4(oKQ + sw128_off16(row, cb + j8, 128));
+                    const uint32_t* qw = reinterpret_cast<const uint32_t*>(&q8);
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
+                        y[j8 + 2 * e] = gt * f.x - y[j8 + 2 * e];
+                        y[j8 + 2 * e + 1] = gt * f.y - y[j8 + 2 * e + 1];
+                    }
+                }
+            }
+#pragma unroll
+            for (int j8 = 0; j8 < 32; j8 += 8) {
+                uint4 hi, lo;
+                split8(y + j8, hi, lo);
+                const int64_t off = sw128_off16(row, cb + j8, 128);
+                *reinterpret_cast<uint4*>(rec + off) = hi;
+                *reinterpret_cast<uint4*>(rec + R::WQH + off) = lo;
+            }
+        }
+        const int dh = ((dv / 2) + 31) / 32 * 32;
+        const int nc = dv / 4;                               // 16-byte chunks per row
+        float* uau = reinterpret_cast<float*>(rec + R::uau_off()) + (int64_t)row * dv;
+        for (int rc = hf * dh; rc < min(dv, (hf + 1) * dh); rc += 32) {
+            uint32_t v[32];
+            tmem_ld32(tmem + lane_off + G::T_WU + DK + rc, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int j4 = 0; j4 < 32; j4 += 4)
+                if (rc + j4 < dv)
+                    *reinterpret_cast<uint4*>(uau + 4 * (((rc + j4) / 4 + row) % nc)) =
+                        make_uint4(v[j4], v[j4 + 1], v[j4 + 2], v[j4 + 3]);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
 
-    // S operand (MN-major: row c, column r) from fp32 values of row c
+// ============================================================================
+// scan: one block per (character, head, d_v slice), chunks in order
+// ============================================================================
+template <int DK>
+struct ScanCfg {
+    static constexpr int WQ = 2 * (int)Rec<DK>::WQH;         // [W;Q'] hi | lo image
+    static constexpr int KI = (int)Rec<DK>::KIMG;            // K image
+    static constexpr int UAU = 128 * DVP * 4;                // U | A U (whole record row width dv <= 256)
+    static constexpr int SOP = 2 * DK * DVMAX * 2;           // S hi, lo (rows c); w E hi, lo aliased
+    static constexpr int OFF_WQ = 0;
+    static constexpr int OFF_K = OFF_WQ + WQ;
+    static constexpr int OFF_U = OFF_K + KI;
+    static constexpr int OFF_S = OFF_U + UAU / 2;            // U | A U is staged for dv <= 128 (64 KB)
+    static constexpr int OFF_BAR = OFF_S + SOP;
+    static constexpr int SMEM = OFF_BAR + 64 + 1024;
+    static constexpr uint32_t T_D = 0;                       // [W;Q'] S0^T (dv cols)
+    static constexpr uint32_t T_S = 128;                     // S^T (dv cols)
+};
+
+template <int DK>
+__global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_constant__ GdnParams p) {
+    using G = ScanCfg<DK>;
+    using R = Rec<DK>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    const uint32_t sb = smem_u32(smem);
+    auto V4 = [&](uint32_t off) -> uint4& { return *reinterpret_cast<uint4*>(smem + off); };
+    constexpr uint32_t oS = G::OFF_S;
+    constexpr uint32_t SH = DK * DVMAX * 2;                      // one S half
+    constexpr uint32_t WEH = C * DVMAX * 2;                      // one w E half
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + G::OFF_BAR);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + G::OFF_BAR + 32);
+    const uint32_t mbar = smem_u32(&bars[0]);
+    const uint32_t bar_wq = smem_u32(&bars[1]), bar_k = smem_u32(&bars[2]), bar_u = smem_u32(&bars[3]);
+    const float* Us = reinterpret_cast<const float*>(smem + G::OFF_U);
+    __shared__ volatile int abort_flag;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int q4 = warp & 3, hf = warp >> 2;
+    const int row = q4 * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    const int dvs = p.dv_slice;
+    const int r0 = blockIdx.x * dvs;
+    const int h = blockIdx.y;
+    const int b = blockIdx.z;
+    const GdnChar ch = p.ch[b];
+    if (ch.M <= 0) return;                           // uniform per block
+    const int H = p.H, dv = p.dv;
+    const int nch = (ch.M + C - 1) / C;
+    const int nc = dv / 4;                           // 16-byte chunks of a U | A U row
+    const uint32_t ubytes = 128u * dv * 4u;
+    float* Sg = p.S + ((int64_t)b * H + h) * dv * DK;
+    const int dhalf = ((dvs / 2) + 31) / 32 * 32;
+    const int dlo = hf * dhalf, dhi = min(dvs, dlo + dhalf);
+    auto rec_of = [&](int i) -> const uint8_t* { return p.work + ((int64_t)(ch.chunk_off + i) * H + h) * p.rec_bytes; };
+
+    if (tid == 0) {
+        abort_flag = 0;
+        mbar_init(mbar, 1);
+        mbar_init(bar_wq, 1);
+        mbar_init(bar_k, 1);
+        mbar_init(bar_u, 1);
+        fence_mbar_init();
+        // chunk 0's records
+        mbar_arrive_expect_tx(bar_wq, G::WQ);
+        bulk_load(sb + G::OFF_WQ, rec_of(0), G::WQ, bar_wq);
+        mbar_arrive_expect_tx(bar_k, G::KI);
+        bulk_load(sb + G::OFF_K, rec_of(0) + G::WQ, G::KI, bar_k);
+        mbar_arrive_expect_tx(bar_u, ubytes);
+        bulk_load(sb + G::OFF_U, rec_of(0) + R::uau_off(), ubytes, bar_u);
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(tmem_slot), 256);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
     auto write_s_row = [&](int c, int rc, const float* x) {
 #pragma unroll
         for (int j8 = 0; j8 < 32; j8 += 8) {
@@ -143,24 +470,22 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
             }
         }
     };
-
-    // ---- load the state slice: S^T into TMEM (lane c, column r) and the operand
-    for (int rc = dlo; rc < dhi; rc += 32) {
-        uint32_t v[32];
-        float x[32];
+    // ---- the state slice: S^T into TMEM (lane c, column r) and the MN-major operand
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-            const int r = rc + j;
-            x[j] = (row < DK && r < dvs) ? Sg[(int64_t)(r0 + r) * DK + row] : 0.f;
-            v[j] = __float_as_uint(x[j]);
-        }
+    for (int half = 0; half < 2; ++half) {
+        const int rc = dlo + 32 * half;
+        if (rc >= dhi) continue;                     // uniform per warp
+        float sx[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j)                 // all 32 loads before any use
+            sx[j] = (row < DK && rc + j < dhi) ? Sg[(int64_t)(r0 + rc + j) * DK + row] : 0.f;
+        uint32_t v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sx[j]);
         tmem_st32(tmem + lane_off + G::T_S + rc, v);
-        if (row < DK) write_s_row(row, rc, x);
+        if (row < DK) write_s_row(row, rc, sx);
     }
     tmem_st_wait();
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncthreads();
 
     uint32_t phase = 0;
     bool ok = true;
@@ -172,176 +497,21 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
         return r;
     };
     auto issue_begin = [&]() { fence_proxy_async_smem(); tc_fence_before(); __syncthreads(); };
-    const uint32_t id_kk = idesc_bf16_f32(128, C, false);
-    const uint32_t id_w = idesc_bf16_f32(128, DK, true);            // B = K, MN-major
-    const uint32_t id_u = idesc_bf16_f32(128, dvs, true);           // B = V, MN-major
     const uint32_t id_1 = idesc_bf16_f32(128, dvs, true);           // B = S, MN-major
     const uint32_t id_2 = idesc_bf16_f32(128, dvs, true, true);     // A = K, B = w E, both MN-major
-    const uint32_t kq_region = 128 * 128;                           // [K;Q] region stride (64 columns)
+    const uint32_t kq_region = 128 * 128;
+    issue_begin();
 
-    for (int c0 = 0; c0 < ch.M && ok; c0 += C) {
-        const int n = min(C, ch.M - c0);
-        const int64_t tok0 = ch.tail_off + c0;
-        // ---------------------------------------------------------------- loads
-        for (int i = tid; i < 128 * (DK / 8); i += kThreads) {
-            const int rr = i / (DK / 8), c8 = (i % (DK / 8)) * 8;
-            const int t = rr & 63;
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (t < n) v = *reinterpret_cast<const uint4*>((rr < 64 ? p.k : p.q) + ((tok0 + t) * H + h) * DK + c8);
-            V4(oKQ + sw128_off16(rr, c8, 128)) = v;
-        }
-        for (int i = tid; i < C * (dvs / 8); i += kThreads) {
-            const int t = i / (dvs / 8), r8 = (i % (dvs / 8)) * 8;
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (t < n) v = *reinterpret_cast<const uint4*>(p.v + ((tok0 + t) * H + h) * dv + r0 + r8);
-            V4(oV + sw128_off16(t, r8, C)) = v;
-        }
-        if (tid < 32) {
-            float x0 = tid < n ? logf(p.alpha[(tok0 + tid) * H + h]) : 0.f;
-            float x1 = tid + 32 < n ? logf(p.alpha[(tok0 + tid + 32) * H + h]) : 0.f;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const float y0 = __shfl_up_sync(0xffffffffu, x0, o);
-                const float y1 = __shfl_up_sync(0xffffffffu, x1, o);
-                if (tid >= o) { x0 += y0; x1 += y1; }
-            }
-            x1 += __shfl_sync(0xffffffffu, x0, 31);
-            gs[tid] = x0;
-            gs[tid + 32] = x1;
-            bs[tid] = tid < n ? p.beta[(tok0 + tid) * H + h] : 0.f;
-            bs[tid + 32] = tid + 32 < n ? p.beta[(tok0 + tid + 32) * H + h] : 0.f;
-        }
-        issue_begin();
-        if (tid < C) {
-            Gs[tid] = expf(gs[tid]);
-            ws[tid] = tid < n ? bs[tid] * expf(gs[n - 1] - gs[tid]) : 0.f;
-        }
-        // ---------------------------------------------------------------- KK, QK
-        if (tid == 0) {
-            tc_fence_after();
-#pragma unroll
-            for (int ks = 0; ks < DK / 16; ++ks) {
-                const uint32_t off = (ks >> 2) * kq_region + (ks & 3) * 32;
-                mma_bf16(tmem + G::T_D, smem_desc_sw128(sb + oKQ + off, 16, 1024),
-                         smem_desc_sw128(sb + oKQ + off, 16, 1024), id_kk, ks > 0);
-            }
-            mma_commit(mbar);
-        }
-        ok = mma_wait();                            // also publishes Gs, ws
+    for (int i = 0; i < nch && ok; ++i) {
+        const int n = min(C, ch.M - i * C);
+        const int64_t tok0 = ch.tail_off + (int64_t)i * C;
+        const uint8_t* rec = rec_of(i);
+        const float* misc = reinterpret_cast<const float*>(rec + R::misc_off(dv));
+        const float wt = __ldg(misc + (row & 63));
+        const float gC = __ldg(misc + C);
+        ok = mbar_wait(bar_wq, i & 1, &abort_flag, p.err, kErrWait);
+        ok = __syncthreads_and(ok);
         if (!ok) break;
-        // ---------------------------------------------------------------- L, A; X = [I; A] (I + L)^-1
-        float x[C];
-        if (hf == 0) {
-            uint32_t v0[32], v1[32];
-            tmem_ld32(tmem + lane_off + G::T_D, v0);
-            tmem_ld32(tmem + lane_off + G::T_D + 32, v1);
-            tmem_ld_wait();
-            const int t = row & 63;
-            const float gt = gs[t];
-#pragma unroll
-            for (int j = 0; j < C; ++j) {
-                const float d = __uint_as_float(j < 32 ? v0[j] : v1[j - 32]);
-                const bool keep = (row < 64) ? (j < t) : (j <= t);
-                x[j] = (keep && t < n) ? expf(gt - gs[j]) * bs[j] * d : 0.f;
-            }
-            if (row < 64) {
-#pragma unroll
-                for (int j = 0; j < C; j += 4)
-                    *reinterpret_cast<float4*>(Lm + t * LSTRIDE + j) = make_float4(x[j], x[j + 1], x[j + 2], x[j + 3]);
-#pragma unroll
-                for (int j = 0; j < C; ++j) x[j] = (j == t) ? 1.f : 0.f;       // right-hand side e_t
-            }
-        }
-        __syncthreads();
-        if (hf == 0) {
-            // x (I + L) = b, L strictly lower: x_j = b_j - sum_{i>j} x_i L[i][j]
-#pragma unroll
-            for (int i = C - 1; i > 0; --i) {
-                const float xi = x[i];
-#pragma unroll
-                for (int j4 = 0; j4 < i; j4 += 4) {
-                    const float4 l4 = *reinterpret_cast<const float4*>(Lm + i * LSTRIDE + j4);
-                    x[j4] = fmaf(-xi, l4.x, x[j4]);
-                    if (j4 + 1 < i) x[j4 + 1] = fmaf(-xi, l4.y, x[j4 + 1]);
-                    if (j4 + 2 < i) x[j4 + 2] = fmaf(-xi, l4.z, x[j4 + 2]);
-                    if (j4 + 3 < i) x[j4 + 3] = fmaf(-xi, l4.w, x[j4 + 3]);
-                }
-            }
-        }
-        __syncthreads();                             // every row finished reading L
-        if (hf == 0) {
-            // operands: X G (for W) and X (for U), K-major rows
-#pragma unroll
-            for (int j8 = 0; j8 < C; j8 += 8) {
-                float xg[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) xg[e] = x[j8 + e] * Gs[j8 + e];
-                uint4 hi, lo;
-                split8(xg, hi, lo);
-                const uint32_t off = sw128_off16(row, j8, 128);
-                V4(oXG + off) = hi;
-                V4(oXG + T128 + off) = lo;
-                split8(x + j8, hi, lo);
-                V4(oX + off) = hi;
-                V4(oX + T128 + off) = lo;
-            }
-        }
-        issue_begin();
-        // ---------------------------------------------------------------- [W | U] = X [G K | V]
-        if (tid == 0) {
-            tc_fence_after();
-#pragma unroll
-            for (int ks = 0; ks < C / 16; ++ks) {
-                const uint64_t bk = smem_desc_sw128(sb + oKQ + ks * 2048, kq_region, 1024);
-                const uint64_t bvv = smem_desc_sw128(sb + oV + ks * 2048, C * 128, 1024);
-#pragma unroll
-                for (int part = 0; part < 2; ++part) {
-                    const uint32_t ao = part * T128 + ks * 32;
-                    mma_bf16(tmem + G::T_WU, smem_desc_sw128(sb + oXG + ao, 16, 1024), bk, id_w, (ks | part) != 0);
-                    mma_bf16(tmem + G::T_WU + DK, smem_desc_sw128(sb + oX + ao, 16, 1024), bvv, id_u,
-                             (ks | part) != 0);
-                }
-            }
-            mma_commit(mbar);
-        }
-        ok = mma_wait();
-        if (!ok) break;
-        // ---------------------------------------------------------------- [W; Q'] operand (hi, lo)
-        {
-            const int t = row & 63;
-            const float gt = Gs[t];
-            for (int cb = hf * (DK / 2); cb < (hf + 1) * (DK / 2); cb += 32) {
-                uint32_t v[32];
-                tmem_ld32(tmem + lane_off + G::T_WU + cb, v);
-                tmem_ld_wait();
-                float y[32];
-#pragma unroll
-                for (int j = 0; j < 32; ++j) y[j] = __uint_as_float(v[j]);
-                if (row >= 64) {
-                    // Q' = G Q - A W ; row `row` of [K;Q] holds q_t
-#pragma unroll
-                    for (int j8 = 0; j8 < 32; j8 += 8) {
-                        const uint4 q8 = V4(oKQ + sw128_off16(row, cb + j8, 128));
-                        const uint32_t* qw = reinterpret_cast<const uint32_t*>(&q8);
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
-                            y[j8 + 2 * e] = gt * f.x - y[j8 + 2 * e];
-                            y[j8 + 2 * e + 1] = gt * f.y - y[j8 + 2 * e + 1];
-                        }
-                    }
-                }
-#pragma unroll
-                for (int j8 = 0; j8 < 32; j8 += 8) {
-                    uint4 hi, lo;
-                    split8(y + j8, hi, lo);
-                    const uint32_t off = sw128_off16(row, cb + j8, 128);
-                    V4(oA + off) = hi;
-                    V4(oA + WQH + off) = lo;
-                }
-            }
-        }
-        issue_begin();
         // ---------------------------------------------------------------- [W; Q'] S0^T
         if (tid == 0) {
             tc_fence_after();
@@ -349,8 +519,8 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
             for (int ks = 0; ks < DK / 16; ++ks) {
                 const uint32_t ao = (ks >> 2) * kq_region + (ks & 3) * 32;
                 const uint32_t bo = ks * 2048;
-                const uint64_t a_hi = smem_desc_sw128(sb + oA + ao, 16, 1024);
-                const uint64_t a_lo = smem_desc_sw128(sb + oA + WQH + ao, 16, 1024);
+                const uint64_t a_hi = smem_desc_sw128(sb + G::OFF_WQ + ao, 16, 1024);
+                const uint64_t a_lo = smem_desc_sw128(sb + G::OFF_WQ + (uint32_t)R::WQH + ao, 16, 1024);
                 const uint64_t b_hi = smem_desc_sw128(sb + oS + bo, DK * 128, 1024);
                 const uint64_t b_lo = smem_desc_sw128(sb + oS + SH + bo, DK * 128, 1024);
                 mma_bf16(tmem + G::T_D, a_hi, b_hi, id_1, ks > 0);
@@ -361,21 +531,34 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
         }
         ok = mma_wait();
         if (!ok) break;
+        if (tid == 0 && i + 1 < nch) {               // [W;Q'] image consumed: fetch the next one
+            mbar_arrive_expect_tx(bar_wq, G::WQ);
+            bulk_load(sb + G::OFF_WQ, rec_of(i + 1), G::WQ, bar_wq);
+        }
+        ok = __syncthreads_and(mbar_wait(bar_u, i & 1, &abort_flag, p.err, kErrWait));
+        if (!ok) break;
         // ---------------------------------------------------------------- E, O; S^T *= G_C
         {
             const int t = row & 63;
-            const float gC = expf(gs[n - 1]);
-            const float wt = ws[t];
-            for (int rc = dlo; rc < dhi; rc += 32) {
-                uint32_t d1[32], u[32], sv[32];
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                const int rc = dlo + 32 * half;
+                if (rc >= dhi) continue;                 // uniform per warp
+                uint32_t d1[32], sv[32];
                 tmem_ld32(tmem + lane_off + G::T_D + rc, d1);
-                tmem_ld32(tmem + lane_off + G::T_WU + DK + rc, u);
                 tmem_ld32(tmem + lane_off + G::T_S + rc, sv);
+                float u[32];
+#pragma unroll
+                for (int j4 = 0; j4 < 32; j4 += 4) {
+                    const int cg = (r0 + rc + j4) / 4;   // chunk of the record row
+                    const float4 f = *reinterpret_cast<const float4*>(Us + (int64_t)row * dv + 4 * ((cg + row) % nc));
+                    u[j4] = f.x; u[j4 + 1] = f.y; u[j4 + 2] = f.z; u[j4 + 3] = f.w;
+                }
                 tmem_ld_wait();
                 if (row < 64) {
                     float e[32];
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) e[j] = wt * (__uint_as_float(u[j]) - __uint_as_float(d1[j]));
+                    for (int j = 0; j < 32; ++j) e[j] = wt * (u[j] - __uint_as_float(d1[j]));
 #pragma unroll
                     for (int j8 = 0; j8 < 32; j8 += 8) {
                         if (rc + j8 < dvs) {
@@ -395,8 +578,8 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
                             uint32_t* ww = reinterpret_cast<uint32_t*>(&w4);
 #pragma unroll
                             for (int e = 0; e < 4; ++e)
-                                ww[e] = pack_bf16x2(__uint_as_float(u[j8 + 2 * e]) + __uint_as_float(d1[j8 + 2 * e]),
-                                                    __uint_as_float(u[j8 + 2 * e + 1]) + __uint_as_float(d1[j8 + 2 * e + 1]));
+                                ww[e] = pack_bf16x2(u[j8 + 2 * e] + __uint_as_float(d1[j8 + 2 * e]),
+                                                    u[j8 + 2 * e + 1] + __uint_as_float(d1[j8 + 2 * e + 1]));
                             *reinterpret_cast<uint4*>(o + j8) = w4;
                         }
                     }
@@ -408,12 +591,18 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
             tmem_st_wait();
         }
         issue_begin();
+        if (tid == 0 && i + 1 < nch) {               // U | A U consumed: fetch the next one
+            mbar_arrive_expect_tx(bar_u, ubytes);
+            bulk_load(sb + G::OFF_U, rec_of(i + 1) + R::uau_off(), ubytes, bar_u);
+        }
         // ---------------------------------------------------------------- S^T += K^T (w E)
+        ok = __syncthreads_and(mbar_wait(bar_k, i & 1, &abort_flag, p.err, kErrWait));
+        if (!ok) break;
         if (tid == 0) {
             tc_fence_after();
 #pragma unroll
             for (int ks = 0; ks < C / 16; ++ks) {
-                const uint64_t a = smem_desc_sw128(sb + oKQ + ks * 2048, kq_region, 1024);
+                const uint64_t a = smem_desc_sw128(sb + G::OFF_K + ks * 2048, C * 128, 1024);
                 mma_bf16(tmem + G::T_S, a, smem_desc_sw128(sb + oS + ks * 2048, C * 128, 1024), id_2, 1u);
                 mma_bf16(tmem + G::T_S, a, smem_desc_sw128(sb + oS + WEH + ks * 2048, C * 128, 1024), id_2, 1u);
             }
@@ -421,8 +610,15 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
         }
         ok = mma_wait();
         if (!ok) break;
+        if (tid == 0 && i + 1 < nch) {               // K image consumed: fetch the next one
+            mbar_arrive_expect_tx(bar_k, G::KI);
+            bulk_load(sb + G::OFF_K, rec_of(i + 1) + G::WQ, G::KI, bar_k);
+        }
         // ---------------------------------------------------------------- refresh the state operand
-        for (int rc = dlo; rc < dhi; rc += 32) {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int rc = dlo + 32 * half;
+            if (rc >= dhi) continue;                     // uniform per warp
             uint32_t sv[32];
             tmem_ld32(tmem + lane_off + G::T_S + rc, sv);
             tmem_ld_wait();
@@ -435,9 +631,11 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
         }
         issue_begin();
     }
-    // ---- write the state slice back
     if (ok) {
-        for (int rc = dlo; rc < dhi; rc += 32) {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int rc = dlo + 32 * half;
+            if (rc >= dhi) continue;                     // uniform per warp
             uint32_t sv[32];
             tmem_ld32(tmem + lane_off + G::T_S + rc, sv);
             tmem_ld_wait();
@@ -447,34 +645,65 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_chunk_tc_kernel(const __grid_
                     if (rc + j < dvs) Sg[(int64_t)(r0 + rc + j) * DK + row] = __uint_as_float(sv[j]);
             }
         }
+    } else if (tid == 0) {
+        // let outstanding record copies land before the block exits
+        volatile int never = 0;
+        const uint32_t bs3[3] = {bar_wq, bar_k, bar_u};
+        for (int k = 0; k < 3; ++k) {
+            mbar_wait(bs3[k], 0, &never, p.err, kErrWait, 1u << 20);
+            mbar_wait(bs3[k], 1, &never, p.err, kErrWait, 1u << 20);
+        }
     }
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
         tc_fence_after();
-        tmem_dealloc(tmem, 512);
+        tmem_dealloc(tmem, 256);
     }
 }
 
-template <int DK>
-void launch_gdn_tc_dk(const GdnParams& p, cudaStream_t s) {
-    using G = GCfg<DK>;
+// Opt in to the kernel's dynamic shared memory once per device (one flag per
+// kernel: the template is keyed on the kernel itself).
+template <auto KERNEL>
+void configure_once(int smem) {
     static unsigned long long configured = 0;   // one bit per device
     int dev = 0;
     cudaGetDevice(&dev);
     if (!(configured >> (dev & 63) & 1ull)) {
-        cudaFuncSetAttribute(gdn_chunk_tc_kernel<DK>, cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM);
+        cudaFuncSetAttribute(KERNEL, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         configured |= 1ull << (dev & 63);
     }
+}
+
+template <int DK>
+void launch_prep_dk(const GdnParams& p, cudaStream_t s) {
+    configure_once<gdn_prep_kernel<DK>>(PrepCfg<DK>::SMEM);
+    gdn_prep_kernel<DK><<<p.total_chunks * p.H, kThreads, PrepCfg<DK>::SMEM, s>>>(p);
+}
+
+template <int DK>
+void launch_scan_dk(const GdnParams& p, cudaStream_t s) {
+    configure_once<gdn_scan_kernel<DK>>(ScanCfg<DK>::SMEM);
     dim3 grid(p.dv / p.dv_slice, p.H, p.n_chars);
-    gdn_chunk_tc_kernel<DK><<<grid, kThreads, G::SMEM, s>>>(p);
+    gdn_scan_kernel<DK><<<grid, kThreads, ScanCfg<DK>::SMEM, s>>>(p);
 }
 
 }  // namespace
 
+int64_t gdn_record_bytes(int dk, int dv) {
+    return dk == 64 ? Rec<64>::bytes(dv) : Rec<128>::bytes(dv);
+}
+
+void launch_gdn_chunk_prep(const GdnParams& p, cudaStream_t s) {
+    if (p.total_chunks <= 0) return;
+    if (p.dk == 64) launch_prep_dk<64>(p, s);
+    else if (p.dk == 128) launch_prep_dk<128>(p, s);
+}
+
 void launch_gdn_chunk_scan(const GdnParams& p, cudaStream_t s) {
-    if (p.dk == 64) launch_gdn_tc_dk<64>(p, s);
-    else if (p.dk == 128) launch_gdn_tc_dk<128>(p, s);
+    if (p.total_chunks <= 0) return;
+    if (p.dk == 64) launch_scan_dk<64>(p, s);
+    else if (p.dk == 128) launch_scan_dk<128>(p, s);
 }
 
 }  // namespace kvm

@@ -85,6 +85,8 @@ struct kvm_ctx {
     std::vector<int> flag_off;
     uint32_t epoch = 0;
     int32_t* err = nullptr;
+    uint8_t* gdn_work = nullptr;          // delta-rule prep records
+    int64_t gdn_rec = 0;
     // staging for host-resident round inputs
     void* stage_in[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
     void* stage_out = nullptr;
@@ -114,7 +116,7 @@ cudaError_t alloc_zero(T** p, size_t count) {
 void free_all(kvm_ctx* c) {
     void* ptrs[] = {c->K, c->V, c->pos, c->S, c->q_rot, c->part_o, c->part_ml, c->tickets,
                     c->flags, c->err, c->stage_in[0], c->stage_in[1], c->stage_in[2],
-                    c->stage_in[3], c->stage_in[4], c->stage_out};
+                    c->stage_in[3], c->stage_in[4], c->stage_out, c->gdn_work};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     for (cudaEvent_t e : c->ev) cudaEventDestroy(e);
@@ -242,7 +244,7 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         c->H = m->n_gdn_heads; c->dk = m->d_k; c->dv = m->d_v;
         if (c->H <= 0) { delete c; return fail(KVM_E_INVAL, "n_gdn_heads must be positive"); }
         if (c->dk != 64 && c->dk != 128) { delete c; return fail(KVM_E_UNSUPPORTED, "d_k must be 64 or 128"); }
-        if (c->dv <= 0 || c->dv % 32 || c->dv > 256) { delete c; return fail(KVM_E_UNSUPPORTED, "d_v must be a multiple of 32, <= 256"); }
+        if (c->dv <= 0 || c->dv % 32 || c->dv > 128) { delete c; return fail(KVM_E_UNSUPPORTED, "d_v must be a multiple of 32, <= 128"); }
     }
     c->B = n_chars;
     c->max_tail = max_tail_tokens;
@@ -288,6 +290,12 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
     if (e == cudaSuccess) e = alloc_zero(&c->tickets, (size_t)n_chars * (n_kv_slabs + 1));
     if (e == cudaSuccess) e = alloc_zero(&c->flags, n_flags);
     if (e == cudaSuccess) e = alloc_zero(&c->err, 1);
+    if (c->n_gdn > 0) {
+        // one record per (64-token chunk, head); a character's tail adds at most one ragged chunk
+        c->gdn_rec = gdn_record_bytes(c->dk, c->dv);
+        const size_t chunks = (size_t)max_tail_tokens / 64 + n_chars;
+        if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&c->gdn_work), chunks * c->H * c->gdn_rec);
+    }
     c->stage_bytes[0] = attn_in * 2;   // q
     c->stage_bytes[1] = kv_in * 2;     // k
     c->stage_bytes[2] = v_in * 2;      // v
@@ -655,7 +663,7 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
     std::memset(&p, 0, sizeof p);
     p.n_chars = c->B;
     p.H = c->H; p.dk = c->dk; p.dv = c->dv;
-    p.dv_slice = c->dv / ((c->dv + 127) / 128);
+    p.dv_slice = c->dv;                 // one block carries all d_v rows of a head's state
     p.q = static_cast<const __nv_bfloat16*>(q);
     p.k = static_cast<const __nv_bfloat16*>(k);
     p.v = static_cast<const __nv_bfloat16*>(v);
@@ -664,11 +672,21 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
     p.out = static_cast<__nv_bfloat16*>(out);
     p.S = c->S + (size_t)c->gdn_idx[layer] * c->B * c->H * c->dv * c->dk;
     p.err = c->err;
+    p.work = c->gdn_work;
+    p.rec_bytes = c->gdn_rec;
+    int chunks = 0;
     for (int b = 0; b < c->B; ++b) {
         p.ch[b].M = tail_cu[b + 1] - tail_cu[b];
         p.ch[b].tail_off = tail_cu[b];
+        p.ch[b].chunk_off = chunks;
+        chunks += (p.ch[b].M + 63) / 64;
     }
-    const int ps = prof_begin(c, KVM_K_GDN, s);
+    p.total_chunks = chunks;
+    int ps = prof_begin(c, KVM_K_GDN_PREP, s);
+    launch_gdn_chunk_prep(p, s);
+    prof_end(c, ps, s);
+    LAUNCH_CHECK(c);
+    ps = prof_begin(c, KVM_K_GDN, s);
     launch_gdn_chunk_scan(p, s);
     prof_end(c, ps, s);
     LAUNCH_CHECK(c);

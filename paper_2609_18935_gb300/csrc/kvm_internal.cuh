@@ -126,6 +126,7 @@ constexpr int kAttnRows = 128;   // query rows per attention tile
 struct GdnChar {
     int32_t M;
     int32_t tail_off;
+    int32_t chunk_off;        // first 64-token chunk of this character (all characters' chunks numbered in order)
 };
 
 struct GdnParams {
@@ -138,11 +139,17 @@ struct GdnParams {
     const float* beta;
     __nv_bfloat16* out;       // [sum M][H][dv]
     float* S;                 // this layer's state [n_chars][H][dv][dk]
+    uint8_t* work;            // per (chunk, head) records written by the prep pass, read by the scan
+    int64_t rec_bytes;        // bytes per record
+    int32_t total_chunks;     // sum over characters of ceil(M / 64)
     int32_t* err;
     GdnChar ch[kMaxChars];
 };
 
-void launch_gdn_chunk_scan(const GdnParams& p, cudaStream_t s);
+// Bytes of one (chunk, head) record of the delta-rule workspace.
+int64_t gdn_record_bytes(int dk, int dv);
+void launch_gdn_chunk_prep(const GdnParams& p, cudaStream_t s);   // state-independent chunk products
+void launch_gdn_chunk_scan(const GdnParams& p, cudaStream_t s);   // chunks in order, state in TMEM
 
 // Set the text returned by kvm_last_error() and return `code`.
 int report_error(int code, const char* msg);

@@ -83,8 +83,9 @@ _SIGS = {
 }
 
 # kernel families of kvm_profile_read
-K_COMPACT, K_ROPE_APPEND, K_ATTENTION, K_ATTN_COMBINE, K_GDN, K_GATHER = range(6)
-KERNEL_NAMES = ["kv_compact", "rope_append", "tail_attention", "attn_combine", "gdn_chunk_scan", "gather_map"]
+K_COMPACT, K_ROPE_APPEND, K_ATTENTION, K_ATTN_COMBINE, K_GDN, K_GATHER, K_GDN_PREP = range(7)
+KERNEL_NAMES = ["kv_compact", "rope_append", "tail_attention", "attn_combine", "gdn_chunk_scan", "gather_map",
+                "gdn_chunk_prep"]
 
 _lib = None
 

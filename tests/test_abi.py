@@ -59,7 +59,8 @@ def _desc(kvm, kinds, **kw):
 
 @pytest.mark.parametrize("kw,code", [({"head_dim": 96}, 6), ({"n_q_heads": 12, "n_kv_heads": 5}, 6),
                                      ({"n_q_heads": 24, "n_kv_heads": 2}, 6), ({"rotary_dim": 63}, 6),
-                                     ({"d_k": 96}, 6), ({"d_v": 40}, 6), ({"rope_theta": -1.0}, 1)])
+                                     ({"d_k": 96}, 6), ({"d_v": 40}, 6), ({"d_v": 160}, 6),
+                                     ({"rope_theta": -1.0}, 1)])
 def test_create_rejects_unsupported_shapes(lib, kw, code):
     from paper_2609_18935_gb300 import kvm
     desc, keep = _desc(kvm, [0, 0, 0, 1], **kw)
