@@ -208,7 +208,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     uint32_t phase = 0;
     bool ok = true;
     auto mma_wait = [&]() -> bool {
-        bool r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait);
+        bool r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait, p.diag, 0x40);
         phase ^= 1;
         r = __syncthreads_and(r);
         tc_fence_after();
@@ -490,7 +490,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     uint32_t phase = 0;
     bool ok = true;
     auto mma_wait = [&]() -> bool {
-        bool r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait);
+        bool r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait, p.diag, 0x50);
         phase ^= 1;
         r = __syncthreads_and(r);
         tc_fence_after();
@@ -509,7 +509,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         const float* misc = reinterpret_cast<const float*>(rec + R::misc_off(dv));
         const float wt = __ldg(misc + (row & 63));
         const float gC = __ldg(misc + C);
-        ok = mbar_wait(bar_wq, i & 1, &abort_flag, p.err, kErrWait);
+        ok = mbar_wait(bar_wq, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x51 + 256 * i);
         ok = __syncthreads_and(ok);
         if (!ok) break;
         // ---------------------------------------------------------------- [W; Q'] S0^T
@@ -535,7 +535,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
             mbar_arrive_expect_tx(bar_wq, G::WQ);
             bulk_load(sb + G::OFF_WQ, rec_of(i + 1), G::WQ, bar_wq);
         }
-        ok = __syncthreads_and(mbar_wait(bar_u, i & 1, &abort_flag, p.err, kErrWait));
+        ok = __syncthreads_and(mbar_wait(bar_u, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x52 + 256 * i));
         if (!ok) break;
         // ---------------------------------------------------------------- E, O; S^T *= G_C
         {
@@ -596,7 +596,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
             bulk_load(sb + G::OFF_U, rec_of(i + 1) + R::uau_off(), ubytes, bar_u);
         }
         // ---------------------------------------------------------------- S^T += K^T (w E)
-        ok = __syncthreads_and(mbar_wait(bar_k, i & 1, &abort_flag, p.err, kErrWait));
+        ok = __syncthreads_and(mbar_wait(bar_k, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x53 + 256 * i));
         if (!ok) break;
         if (tid == 0) {
             tc_fence_after();
@@ -650,8 +650,8 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         volatile int never = 0;
         const uint32_t bs3[3] = {bar_wq, bar_k, bar_u};
         for (int k = 0; k < 3; ++k) {
-            mbar_wait(bs3[k], 0, &never, p.err, kErrWait, 1u << 20);
-            mbar_wait(bs3[k], 1, &never, p.err, kErrWait, 1u << 20);
+            mbar_wait(bs3[k], 0, &never, p.err, kErrWait, nullptr, 0, 20000000ull);
+            mbar_wait(bs3[k], 1, &never, p.err, kErrWait, nullptr, 0, 20000000ull);
         }
     }
     tc_fence_before();

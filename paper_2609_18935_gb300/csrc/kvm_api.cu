@@ -85,6 +85,7 @@ struct kvm_ctx {
     std::vector<int> flag_off;
     uint32_t epoch = 0;
     int32_t* err = nullptr;
+    int32_t* diag = nullptr;              // [16]: where the first expired device wait gave up
     uint8_t* gdn_work = nullptr;          // delta-rule prep records
     int64_t gdn_rec = 0;
     // staging for host-resident round inputs
@@ -116,7 +117,7 @@ cudaError_t alloc_zero(T** p, size_t count) {
 void free_all(kvm_ctx* c) {
     void* ptrs[] = {c->K, c->V, c->pos, c->S, c->q_rot, c->part_o, c->part_ml, c->tickets,
                     c->flags, c->err, c->stage_in[0], c->stage_in[1], c->stage_in[2],
-                    c->stage_in[3], c->stage_in[4], c->stage_out, c->gdn_work};
+                    c->stage_in[3], c->stage_in[4], c->stage_out, c->gdn_work, c->diag};
     for (void* p : ptrs)
         if (p) cudaFree(p);
     for (cudaEvent_t e : c->ev) cudaEventDestroy(e);
@@ -290,6 +291,7 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
     if (e == cudaSuccess) e = alloc_zero(&c->tickets, (size_t)n_chars * (n_kv_slabs + 1));
     if (e == cudaSuccess) e = alloc_zero(&c->flags, n_flags);
     if (e == cudaSuccess) e = alloc_zero(&c->err, 1);
+    if (e == cudaSuccess) e = alloc_zero(&c->diag, 16);
     if (c->n_gdn > 0) {
         // one record per (64-token chunk, head); a character's tail adds at most one ragged chunk
         c->gdn_rec = gdn_record_bytes(c->dk, c->dv);
@@ -606,6 +608,7 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
     p.part_o = c->part_o;
     p.part_ml = c->part_ml;
     p.err = c->err;
+    p.diag = c->diag;
     for (int d = 0; d < c->R / 2; ++d) p.inv_freq[d] = c->inv_freq[d];
     int tiles = 0;
     for (int b = 0; b < c->B; ++b) {
@@ -672,6 +675,7 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
     p.out = static_cast<__nv_bfloat16*>(out);
     p.S = c->S + (size_t)c->gdn_idx[layer] * c->B * c->H * c->dv * c->dk;
     p.err = c->err;
+    p.diag = c->diag;
     p.work = c->gdn_work;
     p.rec_bytes = c->gdn_rec;
     int chunks = 0;
@@ -802,10 +806,13 @@ extern "C" kvm_status kvm_check(kvm_ctx* c, void* stream) {
     int32_t e = 0;
     CUDA_TRY(cudaMemcpy(&e, c->err, 4, cudaMemcpyDeviceToHost));
     if (e) {
+        int32_t d[3] = {0, 0, 0};
+        CUDA_TRY(cudaMemcpy(d, c->diag, sizeof d, cudaMemcpyDeviceToHost));
         CUDA_TRY(cudaMemset(c->err, 0, 4));
+        CUDA_TRY(cudaMemset(c->diag, 0, 16 * sizeof(int32_t)));
         CUDA_TRY(cudaMemset(c->tickets, 0, sizeof(int32_t) * (size_t)c->B * (2 * c->n_attn * c->Hkv + 1)));
-        return fail(KVM_E_DEVICE, "device error word 0x%x (%s%s)", e, (e & kErrBounds) ? "bounds " : "",
-                    (e & kErrWait) ? "wait-timeout" : "");
+        return fail(KVM_E_DEVICE, "device error word 0x%x (%s%s); first expired wait: block %d, tag 0x%x, parity %d",
+                    e, (e & kErrBounds) ? "bounds " : "", (e & kErrWait) ? "wait-timeout" : "", d[0] - 1, d[1], d[2]);
     }
     return KVM_OK;
 }

@@ -111,6 +111,7 @@ struct AttnParams {
     float* part_o;                // [n_items][128][D]
     float* part_ml;               // [n_items][128][2]
     int32_t* err;
+    int32_t* diag;                // first expired wait: block + 1, tag, parity
     double inv_freq[kMaxRotaryHalf];
     AttnChar ch[kMaxChars];
 };
@@ -143,6 +144,7 @@ struct GdnParams {
     int64_t rec_bytes;        // bytes per record
     int32_t total_chunks;     // sum over characters of ceil(M / 64)
     int32_t* err;
+    int32_t* diag;            // first expired wait: block + 1, tag, parity
     GdnChar ch[kMaxChars];
 };
 

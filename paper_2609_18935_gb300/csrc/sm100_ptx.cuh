@@ -42,17 +42,33 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Wait for phase `parity` of a barrier, giving up after `limit` polls or when
-// another role raised *abort.  Returns false if the wait did not complete.
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Wait for phase `parity` of a barrier, giving up after about `limit_ns` of
+// wall time or when another role raised *abort.  Returns false if the wait
+// did not complete; the first wait of a block to expire also records
+// (block, tag, iteration) in diag[0..2] when diag is non-null.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          int* err, int err_bit, uint32_t limit = (1u << 26)) {
+                                          int* err, int err_bit, int* diag = nullptr, int tag = 0,
+                                          uint64_t limit_ns = 250000000ull) {
+    uint64_t t0 = 0;
     for (uint32_t it = 0;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((it & 63) == 63) {
             if (*abort_flag) return false;
-            if (it > limit) {
+            const uint64_t now = globaltimer_ns();
+            if (t0 == 0) t0 = now;
+            else if (now - t0 > limit_ns) {
                 *abort_flag = 1;
                 atomicOr(err, err_bit);
+                if (diag && atomicCAS(diag, 0, (int)blockIdx.x + 1) == 0) {
+                    diag[1] = tag;
+                    diag[2] = (int)parity;
+                }
                 return false;
             }
         }

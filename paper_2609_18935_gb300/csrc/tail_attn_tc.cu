@@ -132,13 +132,13 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
             for (int i = 0; i < n && ok; ++i) {
                 const int st = i & 1;
                 const int row = key_row0 + (kt0 + i) * BN;
-                if (i >= 2) ok = mbar_wait(bar(K_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait);
+                if (i >= 2) ok = mbar_wait(bar(K_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x10 + K_EMPTY + 256 * i);
                 if (!ok) break;
                 mbar_arrive_expect_tx(bar(K_FULL + st), C::KV_BYTES);
                 for (int r = 0; r < C::NREG; ++r)
                     tma_load_2d(sK + st * C::KV_BYTES + r * (BN * 128), &p.tmap_k, r * 64, row, bar(K_FULL + st));
                 issued_k[st] = i;
-                if (i >= 2) ok = mbar_wait(bar(V_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait);
+                if (i >= 2) ok = mbar_wait(bar(V_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x10 + V_EMPTY + 256 * i);
                 if (!ok) break;
                 mbar_arrive_expect_tx(bar(V_FULL + st), C::KV_BYTES);
                 for (int r = 0; r < C::NREG; ++r)
@@ -163,8 +163,8 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
             const uint32_t id_pv = idesc_bf16_f32(BM, D, true);
             auto issue_s = [&](int i) -> bool {
                 const int st = i & 1;
-                if (!mbar_wait(bar(K_FULL + st), (i >> 1) & 1, &abort_flag, p.err, kErrWait)) return false;
-                if (i >= 2 && !mbar_wait(bar(S_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait))
+                if (!mbar_wait(bar(K_FULL + st), (i >> 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x20 + K_FULL + 256 * i)) return false;
+                if (i >= 2 && !mbar_wait(bar(S_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x20 + S_EMPTY + 256 * i))
                     return false;
                 tc_fence_after();
                 const uint32_t kb = sK + st * C::KV_BYTES;
@@ -180,8 +180,8 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
             };
             auto issue_pv = [&](int i) -> bool {
                 const int st = i & 1;
-                if (!mbar_wait(bar(P_FULL), i & 1, &abort_flag, p.err, kErrWait)) return false;
-                if (!mbar_wait(bar(V_FULL + st), (i >> 1) & 1, &abort_flag, p.err, kErrWait)) return false;
+                if (!mbar_wait(bar(P_FULL), i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x20 + P_FULL + 256 * i)) return false;
+                if (!mbar_wait(bar(V_FULL + st), (i >> 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x20 + V_FULL + 256 * i)) return false;
                 tc_fence_after();
                 const uint32_t vb = sV + st * C::KV_BYTES;
 #pragma unroll
@@ -194,7 +194,7 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
                 mma_commit(bar(V_EMPTY + st));
                 return true;
             };
-            bool ok = mbar_wait(bar(Q_FULL), 0, &abort_flag, p.err, kErrWait);
+            bool ok = mbar_wait(bar(Q_FULL), 0, &abort_flag, p.err, kErrWait, p.diag, 0x20 + Q_FULL);
             if (ok) ok = issue_s(0);
             for (int i = 0; i < n && ok; ++i) {
                 if (i + 1 < n) ok = issue_s(i + 1);
@@ -221,7 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
         // waits are made warp-uniform so that an abort never splits a warp
         // before the warp-collective tcgen05.ld / tcgen05.st below
         auto wait_all = [&](int which, uint32_t parity) -> bool {
-            const bool r = mbar_wait(bar(which), parity, &abort_flag, p.err, kErrWait);
+            const bool r = mbar_wait(bar(which), parity, &abort_flag, p.err, kErrWait, p.diag, 0x30 + which);
             return __all_sync(0xffffffffu, r);
         };
         for (int i = 0; i < n && ok; ++i) {
@@ -307,14 +307,16 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
             const int hq = kvh * g + (r % g);
             const int64_t item_row = (int64_t)blockIdx.x * BM + r;
             if (p.n_split == 1) {
-                if (row_valid) {
-                    const float inv = 1.f / l;
-                    __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + hq) * D;
+                // tcgen05.ld is warp-collective (.sync.aligned): every lane
+                // loads, and only lanes of real query rows store
+                const float inv = row_valid ? 1.f / l : 0.f;
+                __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + (row_valid ? tok : 0)) * p.Hq + hq) * D;
 #pragma unroll 1
-                    for (int c0 = 0; c0 < D; c0 += 32) {
-                        uint32_t v[32];
-                        tmem_ld32(tmem + lane_off + C::TMEM_O + c0, v);
-                        tmem_ld_wait();
+                for (int c0 = 0; c0 < D; c0 += 32) {
+                    uint32_t v[32];
+                    tmem_ld32(tmem + lane_off + C::TMEM_O + c0, v);
+                    tmem_ld_wait();
+                    if (row_valid) {
                         uint32_t w[16];
 #pragma unroll
                         for (int e = 0; e < 16; ++e) {
@@ -324,7 +326,8 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
                         }
                         uint4* dst = reinterpret_cast<uint4*>(o + c0);
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) dst[e] = make_uint4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
+                        for (int e = 0; e < 4; ++e)
+                            dst[e] = make_uint4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
                     }
                 }
             } else {

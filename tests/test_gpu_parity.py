@@ -100,6 +100,33 @@ def test_population_varlen_edge_cases():
     _assert_errs(errs, what="edge round 2")
 
 
+@pytest.mark.parametrize("head_dim", [256, 128])
+def test_many_ragged_tiles_without_key_splits(head_dim):
+    """Enough query tiles to fill several waves of the attention grid, so each
+    tile runs with its whole key range (no split-combine), and every
+    character's last tile is ragged: the epilogue writes the output directly
+    with some rows of the tile empty."""
+    import torch
+    from harness import Pair
+    rng = np.random.default_rng(51)
+    n_chars = 16
+    tails = [int(m) for m in rng.integers(60, 330, n_chars)]
+    tails = [m + 1 if m % 16 == 0 else m for m in tails]
+    prefix = [int(n) for n in rng.integers(64, 400, n_chars)]
+    caps = [((n + m + 127) // 128) * 128 for n, m in zip(prefix, tails)]
+    shape = W.ModelShape([W.ATTN], 16, 2, head_dim, 64, 1e4, 1, 64, 32)
+    tiles = sum(2 * ((m + 15) // 16) for m in tails)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    if tiles < 2 * sms:
+        pytest.skip(f"{tiles} query tiles do not fill two waves on {sms} SMs")
+    pair = Pair(shape, prefix, caps, sum(tails), seed_index=51)
+    w = W.Workload("ragged-tiles", 51, shape, prefix, 1)
+    w.plan = [[(0.05, 2, m) for m in tails]]
+    span_cu, sb, se, tails = W.round_plan(w, 0, prefix)
+    errs = pair.run_round(span_cu, sb, se, tails, W.tail_inputs(w, 0, tails))
+    _assert_errs(errs, what=f"ragged tiles D={head_dim}")
+
+
 def test_large_cursor_positions():
     """Positions far beyond the live length (holes only in position space)."""
     from harness import Pair

@@ -225,16 +225,20 @@ def make_workload(name: str, n_layers: int | None = None) -> Workload:
 # ----------------------------------------------------------------------------
 # per-round and prefix inputs
 # ----------------------------------------------------------------------------
-def tail_inputs(w: Workload, rnd: int, tails: list) -> dict:
+def tail_inputs(w: Workload, rnd: int, tails: list, layers=None) -> dict:
     """Inputs of one maintenance round, packed over characters.
 
     tails[b] = M_b.  Returns {layer: dict(q, k, v[, alpha, beta])} with
     q/k/v as bf16 bits [sum M][heads][dim]; alpha/beta fp32 [sum M][heads].
+    `layers` restricts the draw to some layers (each layer has its own seeds,
+    so a layer's values do not depend on which others are drawn).
     """
     s = w.shape
     base = w.index * 1000 + rnd
     out = {}
     for layer, kind in enumerate(s.layer_kind):
+        if layers is not None and layer not in layers:
+            continue
         parts = {"q": [], "k": [], "v": [], "alpha": [], "beta": []}
         for b, m in enumerate(tails):
             sd = (base, b, layer)
