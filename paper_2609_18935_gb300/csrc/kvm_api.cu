@@ -49,7 +49,12 @@ kvm_status fail(kvm_status code, const char* fmt, ...) {
         if (e_ != cudaSuccess) return fail(KVM_E_CUDA, "kernel launch failed: %s", cudaGetErrorString(e_)); \
     } while (0)
 
-constexpr int kItemCap = 1024;      // attention work items that may keep a split partial
+// Persistent attention blocks of a context: one wave on this device, at most
+// kMaxAttnCtas.
+int attention_grid_cap(int num_sms, int head_dim) {
+    return std::max(1, std::min(kMaxAttnCtas, num_sms * attention_ctas_per_sm(head_dim)));
+}
+constexpr int kMinUnitsPerCta = 4;  // smallest share of (query tile, key tile) units per attention block
 
 }  // namespace
 
@@ -286,8 +291,9 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
     if (e == cudaSuccess) e = alloc_zero(&c->pos, c->n_attn ? (size_t)c->T_cap : 0);
     if (e == cudaSuccess) e = alloc_zero(&c->S, (size_t)c->n_gdn * n_chars * c->H * c->dv * c->dk);
     if (e == cudaSuccess) e = alloc_zero(&c->q_rot, c->n_attn ? (size_t)max_tail_tokens * c->Hq * c->D : 0);
-    if (e == cudaSuccess) e = alloc_zero(&c->part_o, c->n_attn ? (size_t)kItemCap * kAttnRows * c->D : 0);
-    if (e == cudaSuccess) e = alloc_zero(&c->part_ml, c->n_attn ? (size_t)kItemCap * kAttnRows * 2 : 0);
+    const size_t part_slots = c->n_attn ? 2 * (size_t)attention_grid_cap(c->num_sms, c->D) : 0;
+    if (e == cudaSuccess) e = alloc_zero(&c->part_o, part_slots * kAttnRows * c->D);
+    if (e == cudaSuccess) e = alloc_zero(&c->part_ml, part_slots * kAttnRows * 2);
     if (e == cudaSuccess) e = alloc_zero(&c->tickets, (size_t)n_chars * (n_kv_slabs + 1));
     if (e == cudaSuccess) e = alloc_zero(&c->flags, n_flags);
     if (e == cudaSuccess) e = alloc_zero(&c->err, 1);
@@ -610,7 +616,10 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
     p.err = c->err;
     p.diag = c->diag;
     for (int d = 0; d < c->R / 2; ++d) p.inv_freq[d] = c->inv_freq[d];
+    // query tiles (character, KV head, tile) and their 64-key tiles
+    const int tpt = p.tok_per_tile;
     int tiles = 0;
+    int64_t units = 0;
     for (int b = 0; b < c->B; ++b) {
         AttnChar& ch = p.ch[b];
         ch.L_prev = c->live[b];
@@ -618,23 +627,44 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
         ch.tail_off = tail_cu[b];
         ch.cap_off = c->cap_off[b];
         ch.p = c->cursor[b];
-        ch.n_qtiles = (ch.M + p.tok_per_tile - 1) / p.tok_per_tile;
+        ch.n_qtiles = (ch.M + tpt - 1) / tpt;
+        ch.tile_off = tiles;
         tiles += c->Hkv * ch.n_qtiles;
+        for (int qt = 0; qt < ch.n_qtiles; ++qt)
+            units += (int64_t)c->Hkv * ((ch.L_prev + std::min(ch.M, (qt + 1) * tpt) + 63) / 64);
     }
-    // key splits: when the query tiles alone leave SMs idle, split each tile's
-    // keys so that the items fill one wave (1 block per SM at head_dim 256,
-    // 2 otherwise)
-    const int wave = c->num_sms * (c->D == 256 ? 1 : 2);
-    int split = 1;
-    if (tiles < wave) split = std::max(1, std::min(16, wave / tiles));
-    while (split > 1 && (size_t)tiles * split > (size_t)kItemCap) --split;
-    p.n_split = split;
-    int items = 0;
-    for (int b = 0; b < c->B; ++b) {
-        p.ch[b].item_off = items;
-        items += c->Hkv * p.ch[b].n_qtiles * split;
+    p.n_tiles = tiles;
+    // stream-K: block cc processes units [cc U / G, (cc + 1) U / G), located
+    // as (query tile, key tile) by one walk over the tiles
+    const int G = (int)std::max<int64_t>(1, std::min<int64_t>(attention_grid_cap(c->num_sms, c->D),
+                                                              units / kMinUnitsPerCta));
+    p.n_ctas = G;
+    {
+        int cc = 0, t = 0;
+        int64_t base = 0;
+        for (int b = 0; b < c->B && cc < G; ++b) {
+            const AttnChar& ch = p.ch[b];
+            for (int h = 0; h < c->Hkv && cc < G; ++h)
+                for (int qt = 0; qt < ch.n_qtiles && cc < G; ++qt, ++t) {
+                    const int nk = (ch.L_prev + std::min(ch.M, (qt + 1) * tpt) + 63) / 64;
+                    while (cc < G && (int64_t)cc * units / G < base + nk) {
+                        p.cta_tile[cc] = t;
+                        p.cta_k[cc] = (int)((int64_t)cc * units / G - base);
+                        ++cc;
+                    }
+                    base += nk;
+                }
+        }
+        p.cta_tile[G] = tiles;
+        p.cta_k[G] = 0;
     }
-    p.n_items = items;
+    // tiles shared by several blocks: each is merged once, from the first
+    // block that starts inside it
+    p.n_split_tiles = 0;
+    for (int cc = 1; cc < G; ++cc)
+        if (p.cta_k[cc] > 0 && !(p.cta_tile[cc - 1] == p.cta_tile[cc] && p.cta_k[cc - 1] > 0))
+            p.split_cb[p.n_split_tiles++] = cc;
+    const bool split_tiles = p.n_split_tiles > 0;
 
     int ps = prof_begin(c, KVM_K_ROPE_APPEND, s);
     launch_rope_append(p, total, s);
@@ -644,9 +674,9 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
     launch_tail_attention(p, s);
     prof_end(c, ps, s);
     LAUNCH_CHECK(c);
-    if (split > 1) {
+    if (split_tiles) {
         ps = prof_begin(c, KVM_K_ATTN_COMBINE, s);
-        launch_attn_combine(p, tiles, s);
+        launch_attn_combine(p, s);
         prof_end(c, ps, s);
         LAUNCH_CHECK(c);
     }

@@ -83,8 +83,13 @@ struct AttnChar {
     int32_t cap_off;      // slot offset of the character in the slabs
     int64_t p;            // cursor: position of tail token 0
     int32_t n_qtiles;     // query tiles per KV head
-    int32_t item_off;     // first work item (tile * split) of this character
+    int32_t tile_off;     // first query tile of this character (tiles ordered character, KV head, tile)
 };
+
+// The attention's work is the list of (query tile, 64-key tile) units, query
+// tiles in order and each tile's key tiles in order; persistent block c
+// processes units [start_c, start_{c+1}), given as (query tile, key tile).
+constexpr int kMaxAttnCtas = 320;
 
 struct AttnParams {
     // TMA maps: rotated q [max_tail][Hq][D] (box 64 x g x 128/g), and every
@@ -95,8 +100,8 @@ struct AttnParams {
     int32_t attn_layer;   // index among attention layers
     int32_t n_chars;
     int32_t Hq, Hkv, D, R, g;
-    int32_t n_split;      // key splits per query tile
-    int32_t n_items;      // total work items
+    int32_t n_tiles;      // query tiles over all characters and KV heads
+    int32_t n_ctas;       // persistent attention blocks
     int32_t tok_per_tile; // tail tokens per 128-row query tile (128 / g)
     float scale_log2;     // log2(e) / sqrt(D)
     int64_t slab_rows;    // rows per (layer, head) slab
@@ -108,17 +113,22 @@ struct AttnParams {
     __nv_bfloat16* V;
     int32_t* pos;                 // [slab_rows]
     __nv_bfloat16* out;           // [sum M][Hq][D]
-    float* part_o;                // [n_items][128][D]
-    float* part_ml;               // [n_items][128][2]
+    float* part_o;                // [2 n_ctas][D / 32][128][32]: partial O of a block's first / last segment
+    float* part_ml;               // [2 n_ctas][128][2]: (reference max in log2 units, sum) of a partial
     int32_t* err;
     int32_t* diag;                // first expired wait: block + 1, tag, parity
     double inv_freq[kMaxRotaryHalf];
+    int32_t cta_tile[kMaxAttnCtas + 1];
+    int32_t cta_k[kMaxAttnCtas + 1];
+    int32_t n_split_tiles;                   // query tiles shared by several blocks
+    int32_t split_cb[kMaxAttnCtas];          // per such tile: the first block that starts inside it
     AttnChar ch[kMaxChars];
 };
 
 void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s);
 void launch_tail_attention(const AttnParams& p, cudaStream_t s);
-void launch_attn_combine(const AttnParams& p, int n_tiles, cudaStream_t s);
+void launch_attn_combine(const AttnParams& p, cudaStream_t s);
+int attention_ctas_per_sm(int head_dim);
 constexpr int kAttnRows = 128;   // query rows per attention tile
 
 // ----------------------------------------------------------------------------

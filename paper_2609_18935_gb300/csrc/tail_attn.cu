@@ -7,9 +7,10 @@
 //                The angle pos * omega_d is formed and reduced modulo 2*pi in
 //                fp64 (positions far beyond the live length stay accurate),
 //                then sin/cos and the rotation run in fp32.
-//  attn_combine : merge the key splits of the attention: each split leaves
-//                an unnormalised accumulator and (reference max in log2
-//                units, sum); one warp per query row.
+//  attn_combine : merge the partials of query tiles that the attention's
+//                persistent blocks split between them: each partial is an
+//                unnormalised accumulator with (reference max in log2 units,
+//                sum); one warp per query row.
 #include "kvm_internal.cuh"
 
 namespace kvm {
@@ -58,48 +59,89 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
     const int D = p.D;
 
     __shared__ float cs[kMaxRotaryHalf], sn[kMaxRotaryHalf];
-    for (int d = threadIdx.x; d < half; d += blockDim.x) {
-        const double ang = (double)pos * p.inv_freq[d];
-        const double r = fma(-rint(ang * (1.0 / kTwoPi)), kTwoPi, ang);   // ang mod 2*pi, |r| <= pi
-        float sv, cv;
-        sincosf((float)r, &sv, &cv);
-        cs[d] = cv;
-        sn[d] = sv;
-    }
-    __syncthreads();
-
     const __nv_bfloat16* qrow = p.q + (int64_t)n * p.Hq * D;
     __nv_bfloat16* qdst = p.q_rot + (int64_t)n * p.Hq * D;
     const __nv_bfloat16* krow = p.k_new + (int64_t)n * p.Hkv * D;
     const __nv_bfloat16* vrow = p.v_new + (int64_t)n * p.Hkv * D;
     if ((half & 7) == 0) {
         // 16-byte groups: group g < half/8 rotates with group g + half/8;
-        // groups from R/8 on are copied
+        // groups from R/8 on are copied.  The first kPre items of each thread
+        // are loaded before the angles are formed, so the loads overlap the
+        // trigonometry.
         const int rot = half / 8, copy = (D - p.R) / 8, per_head = rot + copy;
-        for (int idx = threadIdx.x; idx < (p.Hq + p.Hkv) * per_head; idx += blockDim.x) {
+        const int n_items = (p.Hq + p.Hkv) * per_head;
+        constexpr int kPre = 4;
+        auto src_of = [&](int idx, int& d0, bool& rotated, __nv_bfloat16*& dst) -> const __nv_bfloat16* {
             const int h = idx / per_head, gidx = idx % per_head;
             const bool is_q = h < p.Hq;
             const int hh = is_q ? h : h - p.Hq;
-            const __nv_bfloat16* src = is_q ? qrow + hh * D : krow + hh * D;
-            __nv_bfloat16* dst = is_q ? qdst + hh * D : p.K + ((int64_t)hh * p.slab_rows + slot) * D;
-            if (gidx < rot) {
-                const int d0 = gidx * 8;
-                uint4 a = *reinterpret_cast<const uint4*>(src + d0);
-                uint4 bb = *reinterpret_cast<const uint4*>(src + d0 + half);
-                rotate8(a, bb, cs, sn, d0);
-                *reinterpret_cast<uint4*>(dst + d0) = a;
-                *reinterpret_cast<uint4*>(dst + d0 + half) = bb;
-            } else {
-                const int d0 = p.R + (gidx - rot) * 8;
-                *reinterpret_cast<uint4*>(dst + d0) = *reinterpret_cast<const uint4*>(src + d0);
+            dst = is_q ? qdst + hh * D : p.K + ((int64_t)hh * p.slab_rows + slot) * D;
+            rotated = gidx < rot;
+            d0 = rotated ? gidx * 8 : p.R + (gidx - rot) * 8;
+            return is_q ? qrow + hh * D : krow + hh * D;
+        };
+        uint4 la[kPre], lb[kPre];
+#pragma unroll
+        for (int u = 0; u < kPre; ++u) {
+            const int idx = threadIdx.x + u * blockDim.x;
+            if (idx < n_items) {
+                int d0; bool rotated; __nv_bfloat16* dst;
+                const __nv_bfloat16* src = src_of(idx, d0, rotated, dst);
+                la[u] = *reinterpret_cast<const uint4*>(src + d0);
+                if (rotated) lb[u] = *reinterpret_cast<const uint4*>(src + d0 + half);
             }
         }
+        // v needs no angle: copy it first
         for (int idx = threadIdx.x; idx < p.Hkv * (D / 8); idx += blockDim.x) {
             const int h = idx / (D / 8), d0 = (idx % (D / 8)) * 8;
             *reinterpret_cast<uint4*>(p.V + ((int64_t)h * p.slab_rows + slot) * D + d0) =
                 *reinterpret_cast<const uint4*>(vrow + h * D + d0);
         }
+        for (int d = threadIdx.x; d < half; d += blockDim.x) {
+            const double ang = (double)pos * p.inv_freq[d];
+            const double r = fma(-rint(ang * (1.0 / kTwoPi)), kTwoPi, ang);   // ang mod 2*pi, |r| <= pi
+            float sv, cv;
+            sincosf((float)r, &sv, &cv);
+            cs[d] = cv;
+            sn[d] = sv;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int u = 0; u < kPre; ++u) {
+            const int idx = threadIdx.x + u * blockDim.x;
+            if (idx < n_items) {
+                int d0; bool rotated; __nv_bfloat16* dst;
+                src_of(idx, d0, rotated, dst);
+                if (rotated) {
+                    rotate8(la[u], lb[u], cs, sn, d0);
+                    *reinterpret_cast<uint4*>(dst + d0) = la[u];
+                    *reinterpret_cast<uint4*>(dst + d0 + half) = lb[u];
+                } else {
+                    *reinterpret_cast<uint4*>(dst + d0) = la[u];
+                }
+            }
+        }
+        for (int idx = threadIdx.x + kPre * blockDim.x; idx < n_items; idx += blockDim.x) {
+            int d0; bool rotated; __nv_bfloat16* dst;
+            const __nv_bfloat16* src = src_of(idx, d0, rotated, dst);
+            uint4 a = *reinterpret_cast<const uint4*>(src + d0);
+            if (rotated) {
+                uint4 bb = *reinterpret_cast<const uint4*>(src + d0 + half);
+                rotate8(a, bb, cs, sn, d0);
+                *reinterpret_cast<uint4*>(dst + d0 + half) = bb;
+            }
+            *reinterpret_cast<uint4*>(dst + d0) = a;
+        }
     } else {
+        for (int d = threadIdx.x; d < half; d += blockDim.x) {
+            const double ang = (double)pos * p.inv_freq[d];
+            const double r = fma(-rint(ang * (1.0 / kTwoPi)), kTwoPi, ang);
+            float sv, cv;
+            sincosf((float)r, &sv, &cv);
+            cs[d] = cv;
+            sn[d] = sv;
+        }
+        __syncthreads();
         auto rotated = [&](const __nv_bfloat16* row, int d) -> float {
             const float x = __bfloat162float(row[d]);
             if (d >= p.R) return x;
@@ -118,57 +160,78 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
     if (threadIdx.x == 0) p.pos[slot] = (int32_t)pos;
 }
 
-// Work item -> (character, KV head, query tile, split).
-__device__ __forceinline__ void decode_item(const AttnParams& p, int item, int& b, int& kvh,
-                                            int& qt, int& sp) {
-    int lo = 0, hi = p.n_chars - 1;
-    while (lo < hi) {
-        int mid = (lo + hi + 1) >> 1;
-        if (p.ch[mid].item_off <= item) lo = mid; else hi = mid - 1;
-    }
-    b = lo;
-    int local = item - p.ch[b].item_off;
-    sp = local % p.n_split;
-    local /= p.n_split;
-    qt = local % p.ch[b].n_qtiles;
-    kvh = local / p.ch[b].n_qtiles;
-}
-
-// grid (tiles, kRows / 8): one warp per query row, lanes over head_dim.
+// grid (n_split_tiles, kRows / 4): block (x, y) merges rows 4y .. 4y + 3 of
+// the x-th query tile that several attention blocks share.  Block cb =
+// split_cb[x] is the first to start inside the tile, so its partials are in
+// the slots of blocks c0 = cb - 1 .. c1 (the last block that starts inside the
+// tile): c0's last segment (slot 2 c0 + 1, or 2 c0 when the tile is also c0's
+// first segment) and the first segments 2 c of the others.  The rows' (max,
+// sum) pairs are loaded together into shared memory, the weights
+// 2^(m_q - max) / sum formed once per row, and each thread then owns four
+// columns of one row and reads every partial's piece with independent loads.
+constexpr int kCombineMaxParts = kMaxAttnCtas + 1;
+constexpr int kCombineRows = 4;
 __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant__ AttnParams p) {
-    const int tile = blockIdx.x;
-    const int r = blockIdx.y * 8 + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    int b, kvh, qt, sp;
-    decode_item(p, tile * p.n_split, b, kvh, qt, sp);
-    const AttnChar& c = p.ch[b];
-    const int tok = qt * p.tok_per_tile + r / p.g;
-    if (tok >= c.M) return;
-    const int D = p.D;
-    const int64_t item0 = (int64_t)tile * p.n_split;
-    float ms[16], ws[16];
-    float mx = -INFINITY;
-    for (int s = 0; s < p.n_split; ++s) {
-        ms[s] = p.part_ml[((item0 + s) * kRows + r) * 2];
-        mx = fmaxf(mx, ms[s]);
+    __shared__ float m_s[kCombineRows][kCombineMaxParts];
+    __shared__ float l_s[kCombineRows][kCombineMaxParts];
+    const int cb = p.split_cb[blockIdx.x];
+    const int t = p.cta_tile[cb];
+    const int c0 = cb - 1;
+    int c1 = cb;
+    while (c1 + 1 < p.n_ctas && p.cta_tile[c1 + 1] == t && p.cta_k[c1 + 1] > 0) ++c1;
+    const int slot0 = (p.cta_tile[c0] == t) ? 2 * c0 : 2 * c0 + 1;
+    const int n_parts = c1 - c0 + 1;
+    auto slot_of = [&](int q) -> int64_t { return q == 0 ? slot0 : 2 * (c0 + q); };
+    const int row0 = blockIdx.y * kCombineRows;
+    for (int e = threadIdx.x; e < kCombineRows * n_parts; e += blockDim.x) {
+        const int rr = e / n_parts, q = e % n_parts;
+        const float2 ml = *reinterpret_cast<const float2*>(p.part_ml + (slot_of(q) * kRows + row0 + rr) * 2);
+        m_s[rr][q] = ml.x;
+        l_s[rr][q] = ml.y;
     }
-    float den = 0.f;
-    for (int s = 0; s < p.n_split; ++s) {
-        ws[s] = (ms[s] == -INFINITY) ? 0.f : exp2f(ms[s] - mx);
-        den += ws[s] * p.part_ml[((item0 + s) * kRows + r) * 2 + 1];
-    }
-    const float inv = 1.f / den;
-    const int hq = kvh * p.g + (r % p.g);
-    __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + hq) * D;
-    for (int v4 = lane; v4 < D / 4; v4 += 32) {
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int s = 0; s < p.n_split; ++s) {
-            if (ws[s] == 0.f) continue;
-            const float4 x = *reinterpret_cast<const float4*>(p.part_o + ((item0 + s) * kRows + r) * D + v4 * 4);
-            acc.x += ws[s] * x.x; acc.y += ws[s] * x.y; acc.z += ws[s] * x.z; acc.w += ws[s] * x.w;
+    __syncthreads();
+    if (threadIdx.x < kCombineRows) {
+        const int rr = threadIdx.x;
+        float mx = -INFINITY;
+        for (int q = 0; q < n_parts; ++q) mx = fmaxf(mx, m_s[rr][q]);
+        float den = 0.f;
+        for (int q = 0; q < n_parts; ++q) {
+            const float w = (m_s[rr][q] == -INFINITY) ? 0.f : exp2f(m_s[rr][q] - mx);
+            m_s[rr][q] = w;                                        // the weight replaces the max
+            den += w * l_s[rr][q];
         }
-        const uint2 packed = make_uint2(f2_to_bf2(acc.x * inv, acc.y * inv), f2_to_bf2(acc.z * inv, acc.w * inv));
-        *reinterpret_cast<uint2*>(o + v4 * 4) = packed;
+        const float inv = den > 0.f ? 1.f / den : 0.f;
+        for (int q = 0; q < n_parts; ++q) m_s[rr][q] *= inv;
+    }
+    __syncthreads();
+
+    int lo = 0, hi = p.n_chars - 1;                                // last b with tile_off <= t
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.ch[mid].tile_off <= t) lo = mid; else hi = mid - 1;
+    }
+    const AttnChar& c = p.ch[lo];
+    const int local = t - c.tile_off;
+    const int kvh = local / c.n_qtiles, qt = local % c.n_qtiles;
+    const int D = p.D;
+    const int groups = D / 32;                                     // 32-column groups
+    for (int idx = threadIdx.x; idx < kCombineRows * groups * 8; idx += blockDim.x) {
+        const int q4 = idx & 7;                                    // 4-column piece of the group
+        const int cg = (idx >> 3) % groups;
+        const int rr = (idx >> 3) / groups;
+        const int r = row0 + rr;
+        const int tok = qt * p.tok_per_tile + r / p.g;
+        if (tok >= c.M) continue;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+        for (int q = 0; q < n_parts; ++q) {
+            const float w = m_s[rr][q];
+            const float4 x = *reinterpret_cast<const float4*>(p.part_o + ((slot_of(q) * groups + cg) * kRows + r) * 32 + q4 * 4);
+            acc.x += w * x.x; acc.y += w * x.y; acc.z += w * x.z; acc.w += w * x.w;
+        }
+        const int hq = kvh * p.g + (r % p.g);
+        __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + hq) * D + cg * 32 + q4 * 4;
+        *reinterpret_cast<uint2*>(o) = make_uint2(f2_to_bf2(acc.x, acc.y), f2_to_bf2(acc.z, acc.w));
     }
 }
 
@@ -179,9 +242,9 @@ void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s) {
     rope_append_kernel<<<total_tokens, 128, 0, s>>>(p);
 }
 
-void launch_attn_combine(const AttnParams& p, int n_tiles, cudaStream_t s) {
-    if (n_tiles <= 0 || p.n_split <= 1) return;
-    attn_combine_kernel<<<dim3(n_tiles, kRows / 8), 256, 0, s>>>(p);
+void launch_attn_combine(const AttnParams& p, cudaStream_t s) {
+    if (p.n_split_tiles <= 0) return;
+    attn_combine_kernel<<<dim3(p.n_split_tiles, kRows / kCombineRows), 256, 0, s>>>(p);
 }
 
 }  // namespace kvm

@@ -1,24 +1,45 @@
 // Causal GQA attention of the true tail over the compacted cache (Eq. 3 for a
 // full-attention layer), on the sm_100-family tensor cores.
 //
-// Work item = (character, KV head, 128-row query tile, key split).  The 128
-// rows are (tail token, query head of the GQA group) pairs, token-major, so
-// every K/V tile serves all g heads of the group.  Per item:
-//   warp 0      TMA producer: Q tile once, then K and V tiles of 64 keys into
-//               a two-stage ring (128-byte swizzled, K-major rows of head_dim);
-//   warp 1      allocates TMEM; lane 0 issues tcgen05.mma:
-//                 S_i = Q K_i^T   (M 128, N 64, K D)   -> TMEM, double-buffered
-//                 O  += P_i V_i   (M 128, N D, K 64)   -> TMEM accumulator
-//               S_{i+1} is issued before PV_i so it overlaps the softmax of i;
-//   warps 2-5   one query row per thread: read S_i from TMEM, mask, online
-//               softmax in base 2 with lazy rescaling (the running reference
-//               max moves only when a score exceeds it by more than 2^8, and
-//               then the O row in TMEM is rescaled), write P_i as bf16 into
-//               shared memory in the MMA's swizzled K-major layout; finally
-//               read O, normalise and store (or store the partial for the
-//               split-combine).
-// Every mbarrier wait is bounded; on expiry the block raises an abort flag,
-// records kErrWait, drains its own copies and MMAs, frees TMEM and returns.
+// Query tiles have 128 rows = (tail token, query head of one GQA group) pairs,
+// token-major, so each K/V tile serves all g heads of the group.  The work is
+// the list of (query tile, 64-key tile) units; it is cut into equal contiguous
+// ranges, one per persistent block (stream-K).  A block's range covers whole
+// query tiles, whose outputs it normalises and stores directly, and at most
+// one partial tile at each end, whose unnormalised accumulator goes to a
+// workspace slot (2c for block c's first segment, 2c + 1 for its last) for
+// attn_combine.
+//
+// Roles of a block (384 threads):
+//   warps 0, 11 TMA producers: lane 0 of warp 0 streams the K tiles, lane 0
+//               of warp 11 the V tiles of each segment's keys, each through a
+//               three-stage ring (64 keys x D, 128-byte swizzle); separate
+//               warps keep the two rings from waiting on each other;
+//   warp 1      allocates TMEM; lane 0 issues S_j = Q K_j^T (tcgen05.mma,
+//               M 128, N 64, K D, Q read from TMEM) into two TMEM buffers;
+//   warp 10     lane 0 issues O += P_j V_j (M 128, N D, K 64) into the TMEM
+//               accumulator.  Two issuers keep the S stream running ahead of
+//               the softmax while the PV stream follows it;
+//   warps 2-9   softmax: each query row is shared by the two warps that see
+//               its TMEM lane quarter (warp w reads lanes 32 (w mod 4) ..),
+//               one per 32-key half of S_j.  They stage the segment's Q tile
+//               in TMEM (the next segment's as soon as the last S of the
+//               current one has landed), exchange row maxima through shared
+//               memory and a pair barrier, keep an online softmax in base 2
+//               with lazy rescaling (the reference max moves only when a
+//               score exceeds it by more than 2^8; the O row is then rescaled
+//               in TMEM, each half its half of the columns) and write P_j as
+//               bf16 into one of two shared buffers in the MMA's swizzled
+//               K-major layout, so that the softmax of tile j+1 does not wait
+//               for PV_j.  At the end of a segment each half stores its half
+//               of the O columns.
+// Q lives in TMEM rather than shared memory: S_j then reads only K_j from
+// shared memory, and the space goes to a third K and V stage.
+// Every mbarrier wait is bounded in time.  On expiry the block raises an
+// abort flag and records kErrWait: the producers and the MMA issuer stop
+// issuing, the softmax warps run their loops to the end without waiting (so
+// that their pair barriers stay matched), and every copy and MMA already
+// issued completes before TMEM and shared memory are released.
 #include "kvm_internal.cuh"
 #include "sm100_ptx.cuh"
 
@@ -27,86 +48,112 @@ namespace {
 
 using namespace ptx;
 
-constexpr int BM = 128;          // query rows per tile
-constexpr int BN = 64;           // keys per K/V tile
-constexpr int kThreads = 192;    // 6 warps
+constexpr int BM = 128;                       // query rows per tile
+constexpr int BN = 64;                        // keys per K/V tile
+constexpr int kSoftmaxThreads = 256;          // warps 2-9
+constexpr int kThreads = 64 + kSoftmaxThreads + 64;   // + warp 10 (PV issuer), warp 11 (V producer)
+constexpr int kPvWarp = 10;
+constexpr int kVWarp = 11;
 
-enum Bar { Q_FULL = 0, K_FULL = 1, K_EMPTY = 3, V_FULL = 5, V_EMPTY = 7, S_FULL = 9, S_EMPTY = 11,
-           P_FULL = 13, PV_DONE = 14, O_FINAL = 15, N_BARS = 16 };
+constexpr int STAGES = 3;                     // K and V ring depth
+
+enum Bar { K_FULL = 0, K_EMPTY = 3, V_FULL = 6, V_EMPTY = 9, S_FULL = 12, S_EMPTY = 14, P_FULL = 16,
+           PV_DONE = 18, Q_FULL = 20, O_FINAL = 21, O_EMPTY = 22, DRAIN_S = 23, DRAIN_PV = 24, N_BARS = 25 };
 
 template <int D>
 struct Cfg {
     static constexpr int NREG = D / 64;                    // 64-column (128-byte) regions
-    static constexpr int Q_BYTES = BM * D * 2;
+    static constexpr int HALF = D / 2;                     // O columns per softmax half
     static constexpr int KV_BYTES = BN * D * 2;
     static constexpr int P_BYTES = BM * BN * 2;
-    static constexpr int OFF_Q = 0;
-    static constexpr int OFF_K = OFF_Q + Q_BYTES;
-    static constexpr int OFF_V = OFF_K + 2 * KV_BYTES;
-    static constexpr int OFF_P = OFF_V + 2 * KV_BYTES;
-    static constexpr int OFF_BAR = OFF_P + P_BYTES;
-    static constexpr int USED = OFF_BAR + N_BARS * 8 + 16;
-    // D = 64 would fit three blocks per SM by shared memory but TMEM holds two
-    static constexpr int SMEM = (USED + 1024 > 80 * 1024 || D != 64) ? USED + 1024 : 80 * 1024;
+    static constexpr int OFF_K = 0;
+    static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
+    static constexpr int OFF_P = OFF_V + STAGES * KV_BYTES;
+    static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+    static constexpr int OFF_SLOT = OFF_BAR + N_BARS * 8;  // TMEM base address
+    static constexpr int OFF_ABORT = OFF_SLOT + 4;
+    static constexpr int OFF_X = (OFF_ABORT + 4 + 15) / 16 * 16;   // float [2][2][BM] row exchange
+    static constexpr int USED = OFF_X + 2 * 2 * BM * 4;
+    // head_dim 256 leaves no room to align the base up: a block without static
+    // shared variables gets a 1024-aligned dynamic base (checked at run time)
+    static constexpr int SLACK = (D == 256) ? 0 : 1024;
+    static constexpr int SMEM = USED + SLACK;
     static constexpr uint32_t TMEM_S = 0;                  // two S buffers of BN columns
     static constexpr uint32_t TMEM_O = 2 * BN;             // D columns
-    static constexpr uint32_t TMEM_COLS = (2 * BN + D <= 256) ? 256 : 512;
+    static constexpr uint32_t TMEM_Q = 2 * BN + D;         // D / 2 columns: Q as bf16 pairs
+    static constexpr uint32_t TMEM_COLS = (TMEM_Q + D / 2 <= 256) ? 256 : 512;
+};
+static_assert(Cfg<256>::SMEM <= 232448, "shared memory of the head_dim 256 attention");
+static_assert(Cfg<256>::TMEM_Q + 128 <= 512, "TMEM of the head_dim 256 attention");
+
+struct Tile {
+    int b, kvh, qt, nk, tok0, tok_end;
 };
 
-__device__ __forceinline__ void decode_item(const AttnParams& p, int item, int& b, int& kvh, int& qt, int& sp) {
-    int lo = 0, hi = p.n_chars - 1;
+// Query tile t -> (character, KV head, tile within the head) and its number
+// of 64-key tiles (every surviving entry plus the tail up to its last token).
+__device__ __forceinline__ Tile decode_tile(const AttnParams& p, int t) {
+    int lo = 0, hi = p.n_chars - 1;               // last b with tile_off <= t
     while (lo < hi) {
-        int mid = (lo + hi + 1) >> 1;
-        if (p.ch[mid].item_off <= item) lo = mid; else hi = mid - 1;
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.ch[mid].tile_off <= t) lo = mid; else hi = mid - 1;
     }
-    b = lo;
-    int local = item - p.ch[b].item_off;
-    sp = local % p.n_split;
-    local /= p.n_split;
-    qt = local % p.ch[b].n_qtiles;
-    kvh = local / p.ch[b].n_qtiles;
+    Tile r;
+    r.b = lo;
+    const AttnChar& c = p.ch[lo];
+    const int local = t - c.tile_off;
+    r.kvh = local / c.n_qtiles;
+    r.qt = local % c.n_qtiles;
+    r.tok0 = r.qt * p.tok_per_tile;
+    r.tok_end = min(c.M, r.tok0 + p.tok_per_tile);
+    r.nk = (c.L_prev + r.tok_end + BN - 1) / BN;
+    return r;
 }
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __grid_constant__ AttnParams p) {
     using C = Cfg<D>;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = smem_raw;
+    if (C::SLACK) {
+        smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    } else if (smem_u32(smem_raw) & 1023u) {
+        if (threadIdx.x == 0) atomicOr(p.err, kErrBounds);
+        return;                                    // uniform: before any barrier or TMEM use
+    }
     const uint32_t sbase = smem_u32(smem);
-    const uint32_t sQ = sbase + C::OFF_Q, sK = sbase + C::OFF_K, sV = sbase + C::OFF_V, sP = sbase + C::OFF_P;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + N_BARS * 8);
-    auto bar = [&](int i) { return smem_u32(&bars[i]); };
-    __shared__ volatile int abort_flag;
+    const uint32_t sK = sbase + C::OFF_K, sV = sbase + C::OFF_V, sP = sbase + C::OFF_P;
+    auto bar = [&](int i) -> uint32_t { return sbase + C::OFF_BAR + 8u * i; };
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_SLOT);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_ABORT);
+    float* xch = reinterpret_cast<float*>(smem + C::OFF_X);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    int b, kvh, qt, sp;
-    decode_item(p, blockIdx.x, b, kvh, qt, sp);
-    const AttnChar& c = p.ch[b];
+    const int cta = blockIdx.x;
     const int g = p.g;
-    const int tok0 = qt * p.tok_per_tile;
-    const int tok_end = min(c.M, tok0 + p.tok_per_tile);
-    const int n_keys = c.L_prev + tok_end;
-    const int kt_total = (n_keys + BN - 1) / BN;
-    const int kt0 = (int)((int64_t)sp * kt_total / p.n_split);
-    const int kt1 = (int)((int64_t)(sp + 1) * kt_total / p.n_split);
-    const int n = kt1 - kt0;
-    const int key_row0 = (p.attn_layer * p.Hkv + kvh) * (int)p.slab_rows + c.cap_off;
+    const int t_begin = p.cta_tile[cta], k_begin = p.cta_k[cta];
+    const int t_end = p.cta_tile[cta + 1], k_end = p.cta_k[cta + 1];
+    auto more = [&](int t, int k) { return t < t_end || (t == t_end && k < k_end); };
 
     if (tid == 0) {
-        abort_flag = 0;
-        mbar_init(bar(Q_FULL), 1);
-        for (int s = 0; s < 2; ++s) {
+        *abort_flag = 0;
+        for (int s = 0; s < STAGES; ++s) {
             mbar_init(bar(K_FULL + s), 1);
             mbar_init(bar(K_EMPTY + s), 1);
             mbar_init(bar(V_FULL + s), 1);
             mbar_init(bar(V_EMPTY + s), 1);
-            mbar_init(bar(S_FULL + s), 1);
-            mbar_init(bar(S_EMPTY + s), 128);
         }
-        mbar_init(bar(P_FULL), 128);
-        mbar_init(bar(PV_DONE), 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(bar(S_FULL + s), 1);
+            mbar_init(bar(S_EMPTY + s), kSoftmaxThreads);
+            mbar_init(bar(P_FULL + s), kSoftmaxThreads);
+            mbar_init(bar(PV_DONE + s), 1);
+        }
+        mbar_init(bar(Q_FULL), kSoftmaxThreads);
         mbar_init(bar(O_FINAL), 1);
+        mbar_init(bar(O_EMPTY), kSoftmaxThreads);
+        mbar_init(bar(DRAIN_S), 1);
+        mbar_init(bar(DRAIN_PV), 1);
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -118,205 +165,278 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ producer
-        if (lane == 0 && n > 0) {
-            prefetch_tmap(&p.tmap_q);
-            prefetch_tmap(&p.tmap_k);
-            prefetch_tmap(&p.tmap_v);
-            mbar_arrive_expect_tx(bar(Q_FULL), C::Q_BYTES);
-            for (int r = 0; r < C::NREG; ++r)
-                tma_load_3d(sQ + r * (BM * 128), &p.tmap_q, r * 64, kvh * g, c.tail_off + tok0, bar(Q_FULL));
-            int issued_k[2] = {-1, -1}, issued_v[2] = {-1, -1};
+    // copies issued by a producer lane (for the drain after an abort)
+    int last_load[STAGES] = {-1, -1, -1};
+
+    if (warp == 0 || warp == kVWarp) {
+        // ------------------------------------------------------------ producers: warp 0 K, warp 11 V
+        if (lane == 0) {
+            const bool is_k = warp == 0;
+            const CUtensorMap* map = is_k ? &p.tmap_k : &p.tmap_v;
+            const uint32_t ring = is_k ? sK : sV;
+            const int full = is_k ? K_FULL : V_FULL, empty = is_k ? K_EMPTY : V_EMPTY;
+            prefetch_tmap(map);
             bool ok = true;
-            for (int i = 0; i < n && ok; ++i) {
-                const int st = i & 1;
-                const int row = key_row0 + (kt0 + i) * BN;
-                if (i >= 2) ok = mbar_wait(bar(K_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x10 + K_EMPTY + 256 * i);
-                if (!ok) break;
-                mbar_arrive_expect_tx(bar(K_FULL + st), C::KV_BYTES);
-                for (int r = 0; r < C::NREG; ++r)
-                    tma_load_2d(sK + st * C::KV_BYTES + r * (BN * 128), &p.tmap_k, r * 64, row, bar(K_FULL + st));
-                issued_k[st] = i;
-                if (i >= 2) ok = mbar_wait(bar(V_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x10 + V_EMPTY + 256 * i);
-                if (!ok) break;
-                mbar_arrive_expect_tx(bar(V_FULL + st), C::KV_BYTES);
-                for (int r = 0; r < C::NREG; ++r)
-                    tma_load_2d(sV + st * C::KV_BYTES + r * (BN * 128), &p.tmap_v, r * 64, row, bar(V_FULL + st));
-                issued_v[st] = i;
-            }
-            if (abort_flag) {
-                // drain this block's own copies before the block exits
-                volatile int never = 0;
-                mbar_wait(bar(Q_FULL), 0, &never, p.err, kErrWait);
-                for (int s = 0; s < 2; ++s) {
-                    if (issued_k[s] >= 0) mbar_wait(bar(K_FULL + s), (issued_k[s] >> 1) & 1, &never, p.err, kErrWait);
-                    if (issued_v[s] >= 0) mbar_wait(bar(V_FULL + s), (issued_v[s] >> 1) & 1, &never, p.err, kErrWait);
+            int j = 0;
+            for (int t = t_begin, k = k_begin; ok && more(t, k); ++t, k = 0) {
+                const Tile T = decode_tile(p, t);
+                const AttnChar& ch = p.ch[T.b];
+                const int k1 = (t == t_end) ? k_end : T.nk;
+                const int key_row0 = (p.attn_layer * p.Hkv + T.kvh) * (int)p.slab_rows + ch.cap_off;
+                for (int kt = k; kt < k1; ++kt, ++j) {
+                    const int st = j % STAGES;
+                    if (j >= STAGES)
+                        ok = mbar_wait(bar(empty + st), (j / STAGES - 1) & 1, abort_flag, p.err, kErrWait, p.diag,
+                                       (is_k ? 0x12 : 0x13) + 256 * j);
+                    if (!ok) break;
+                    mbar_arrive_expect_tx(bar(full + st), C::KV_BYTES);
+                    for (int r = 0; r < C::NREG; ++r)
+                        tma_load_2d(ring + st * C::KV_BYTES + r * (BN * 128), map, r * 64, key_row0 + kt * BN, bar(full + st));
+                    last_load[st] = j;
                 }
             }
         }
         __syncwarp();
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0 && n > 0) {
+        // ------------------------------------------------------------ S issuer
+        if (lane == 0) {
             const uint32_t id_qk = idesc_bf16_f32(BM, BN, false);
-            const uint32_t id_pv = idesc_bf16_f32(BM, D, true);
-            auto issue_s = [&](int i) -> bool {
-                const int st = i & 1;
-                if (!mbar_wait(bar(K_FULL + st), (i >> 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x20 + K_FULL + 256 * i)) return false;
-                if (i >= 2 && !mbar_wait(bar(S_EMPTY + st), ((i >> 1) - 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x20 + S_EMPTY + 256 * i))
-                    return false;
-                tc_fence_after();
-                const uint32_t kb = sK + st * C::KV_BYTES;
+            const uint64_t k_desc0 = smem_desc_sw128(sK, 16, 1024);   // + (byte offset >> 4) per operand
+            bool ok = true;
+            int j = 0, seg = 0;
+            for (int t = t_begin, k = k_begin; ok && more(t, k); ++t, k = 0, ++seg) {
+                const Tile T = decode_tile(p, t);
+                const int n = ((t == t_end) ? k_end : T.nk) - k;
+                ok = mbar_wait(bar(Q_FULL), seg & 1, abort_flag, p.err, kErrWait, p.diag, 0x21 + 256 * seg);
+                for (int i = 0; i < n && ok; ++i, ++j) {
+                    const int sb = j & 1, st = j % STAGES;
+                    ok = mbar_wait(bar(K_FULL + st), (j / STAGES) & 1, abort_flag, p.err, kErrWait, p.diag, 0x22 + 256 * j);
+                    if (ok && j >= 2)
+                        ok = mbar_wait(bar(S_EMPTY + sb), ((j >> 1) - 1) & 1, abort_flag, p.err, kErrWait, p.diag,
+                                       0x23 + 256 * j);
+                    if (!ok) break;
+                    tc_fence_after();
+                    const uint64_t kd = k_desc0 + (uint64_t)((st * C::KV_BYTES) >> 4);
+                    const uint32_t d = tmem + C::TMEM_S + sb * BN;
 #pragma unroll
-                for (int ks = 0; ks < D / 16; ++ks) {
-                    const uint64_t ad = smem_desc_sw128(sQ + (ks >> 2) * (BM * 128) + (ks & 3) * 32, 16, 1024);
-                    const uint64_t bd = smem_desc_sw128(kb + (ks >> 2) * (BN * 128) + (ks & 3) * 32, 16, 1024);
-                    mma_bf16(tmem + C::TMEM_S + st * BN, ad, bd, id_qk, ks > 0);
+                    for (int ks = 0; ks < D / 16; ++ks)
+                        mma_bf16_ts(d, tmem + C::TMEM_Q + ks * 8, kd + (uint64_t)((((ks >> 2) * (BN * 128)) + (ks & 3) * 32) >> 4),
+                                    id_qk, ks > 0);
+                    mma_commit(bar(S_FULL + sb));
+                    mma_commit(bar(K_EMPTY + st));
                 }
-                mma_commit(bar(S_FULL + st));
-                mma_commit(bar(K_EMPTY + st));
-                return true;
-            };
-            auto issue_pv = [&](int i) -> bool {
-                const int st = i & 1;
-                if (!mbar_wait(bar(P_FULL), i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x20 + P_FULL + 256 * i)) return false;
-                if (!mbar_wait(bar(V_FULL + st), (i >> 1) & 1, &abort_flag, p.err, kErrWait, p.diag, 0x20 + V_FULL + 256 * i)) return false;
-                tc_fence_after();
-                const uint32_t vb = sV + st * C::KV_BYTES;
-#pragma unroll
-                for (int ks = 0; ks < BN / 16; ++ks) {
-                    const uint64_t ad = smem_desc_sw128(sP + ks * 32, 16, 1024);
-                    const uint64_t bd = smem_desc_sw128(vb + ks * 16 * 128, BN * 128, 1024);
-                    mma_bf16(tmem + C::TMEM_O, ad, bd, id_pv, (i > 0 || ks > 0) ? 1u : 0u);
-                }
-                mma_commit(bar(PV_DONE));
-                mma_commit(bar(V_EMPTY + st));
-                return true;
-            };
-            bool ok = mbar_wait(bar(Q_FULL), 0, &abort_flag, p.err, kErrWait, p.diag, 0x20 + Q_FULL);
-            if (ok) ok = issue_s(0);
-            for (int i = 0; i < n && ok; ++i) {
-                if (i + 1 < n) ok = issue_s(i + 1);
-                if (ok) ok = issue_pv(i);
             }
-            // every MMA issued by this thread completes before O_FINAL arrives
-            mma_commit(bar(O_FINAL));
+            // every MMA issued by this thread completes before TMEM is released
+            mma_commit(bar(DRAIN_S));
             volatile int never = 0;
-            mbar_wait(bar(O_FINAL), 0, &never, p.err, kErrWait);
+            mbar_wait(bar(DRAIN_S), 0, &never, p.err, kErrWait, nullptr, 0, 1000000000ull);
+        }
+        __syncwarp();
+    } else if (warp == kPvWarp) {
+        // ------------------------------------------------------------ PV issuer
+        if (lane == 0) {
+            const uint32_t id_pv = idesc_bf16_f32(BM, D, true);
+            const uint64_t p_desc0 = smem_desc_sw128(sP, 16, 1024);
+            const uint64_t v_desc0 = smem_desc_sw128(sV, BN * 128, 1024);
+            bool ok = true;
+            int j = 0, seg = 0;
+            for (int t = t_begin, k = k_begin; ok && more(t, k); ++t, k = 0, ++seg) {
+                const Tile T = decode_tile(p, t);
+                const int n = ((t == t_end) ? k_end : T.nk) - k;
+                for (int i = 0; i < n && ok; ++i, ++j) {
+                    const int pb = j & 1, st = j % STAGES;
+                    ok = mbar_wait(bar(P_FULL + pb), (j >> 1) & 1, abort_flag, p.err, kErrWait, p.diag, 0x24 + 256 * j);
+                    if (ok)
+                        ok = mbar_wait(bar(V_FULL + st), (j / STAGES) & 1, abort_flag, p.err, kErrWait, p.diag, 0x25 + 256 * j);
+                    // the previous segment's O has been read out before it is overwritten
+                    if (ok && i == 0 && seg > 0)
+                        ok = mbar_wait(bar(O_EMPTY), (seg - 1) & 1, abort_flag, p.err, kErrWait, p.diag, 0x26 + 256 * seg);
+                    if (!ok) break;
+                    tc_fence_after();
+                    const uint64_t pd = p_desc0 + (uint64_t)((pb * C::P_BYTES) >> 4);
+                    const uint64_t vd = v_desc0 + (uint64_t)((st * C::KV_BYTES) >> 4);
+#pragma unroll
+                    for (int ks = 0; ks < BN / 16; ++ks)
+                        mma_bf16(tmem + C::TMEM_O, pd + (uint64_t)((ks * 32) >> 4), vd + (uint64_t)((ks * 16 * 128) >> 4), id_pv,
+                                 (i > 0 || ks > 0) ? 1u : 0u);
+                    mma_commit(bar(PV_DONE + pb));
+                    mma_commit(bar(V_EMPTY + st));
+                }
+                if (ok) mma_commit(bar(O_FINAL));
+            }
+            mma_commit(bar(DRAIN_PV));
+            volatile int never = 0;
+            mbar_wait(bar(DRAIN_PV), 0, &never, p.err, kErrWait, nullptr, 0, 1000000000ull);
         }
         __syncwarp();
     } else {
         // ------------------------------------------------------------ softmax + epilogue
-        const int quarter = warp & 3;                    // TMEM lanes 32*quarter .. +31
-        const int r = quarter * 32 + lane;               // query row of this thread
+        const int half = (warp - 2) >> 2;                  // key columns 32 half .. +31 of S
+        const int quarter = warp & 3;                      // TMEM lanes 32 quarter .. +31
+        const int r = quarter * 32 + lane;                 // query row of this thread
         const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-        const int tok = tok0 + r / g;
-        const bool row_valid = tok < c.M;
-        const int lim = c.L_prev + min(tok, c.M - 1) + 1;     // keys [0, lim) are visible
+        const int pair_bar = 1 + quarter;
         const float sl = p.scale_log2;
-        float mr = -INFINITY;                            // reference max, log2 units
-        float l = 0.f;
-        bool ok = true;
-        // waits are made warp-uniform so that an abort never splits a warp
-        // before the warp-collective tcgen05.ld / tcgen05.st below
-        auto wait_all = [&](int which, uint32_t parity) -> bool {
-            const bool r = mbar_wait(bar(which), parity, &abort_flag, p.err, kErrWait, p.diag, 0x30 + which);
-            return __all_sync(0xffffffffu, r);
+        // waits do not change the control flow (the pair barriers must stay
+        // matched); after an abort they return at once and the results are
+        // discarded
+        auto wait_all = [&](int which, uint32_t parity, int tag) {
+            __syncwarp();
+            mbar_wait(bar(which), parity, abort_flag, p.err, kErrWait, p.diag, tag);
+            __syncwarp();
         };
-        for (int i = 0; i < n && ok; ++i) {
-            const int st = i & 1;
-            ok = wait_all(S_FULL + st, (i >> 1) & 1);
-            if (!ok) break;
-            tc_fence_after();
-            uint32_t sa[32], sb[32];
-            tmem_ld32(tmem + lane_off + C::TMEM_S + st * BN, sa);
-            tmem_ld32(tmem + lane_off + C::TMEM_S + st * BN + 32, sb);
-            tmem_ld_wait();
-            tc_fence_before();
-            mbar_arrive(bar(S_EMPTY + st));
-            float s[64];
+        // Q tile of query tile t into TMEM: this thread's half of row r (D / 2
+        // bf16 = D / 4 columns); rows past the character's tail are zero
+        auto stage_q = [&](int t) {
+            const Tile T = decode_tile(p, t);
+            const AttnChar& ch = p.ch[T.b];
+            const int tok = T.tok0 + r / g;
+            constexpr int W = D / 4;                       // 32-bit words of this half
+            uint4 v[W / 4];
+            const uint4* src = reinterpret_cast<const uint4*>(
+                p.q_rot + ((int64_t)(ch.tail_off + tok) * p.Hq + T.kvh * g + (r % g)) * D + half * (D / 2));
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                s[j] = __uint_as_float(sa[j]);
-                s[32 + j] = __uint_as_float(sb[j]);
-            }
-            const int key0 = (kt0 + i) * BN;
-            if (key0 + BN > lim) {
+            for (int e = 0; e < W / 4; ++e) v[e] = tok < ch.M ? src[e] : make_uint4(0, 0, 0, 0);
+            const uint32_t* w = reinterpret_cast<const uint32_t*>(v);
+            if constexpr (W >= 32) {
 #pragma unroll
-                for (int j = 0; j < 64; ++j)
-                    if (key0 + j >= lim) s[j] = -INFINITY;
-            }
-            float mx = s[0];
+                for (int c0 = 0; c0 < W; c0 += 32) {
+                    uint32_t x[32];
 #pragma unroll
-            for (int j = 1; j < 64; ++j) mx = fmaxf(mx, s[j]);
-            const float mx2 = mx * sl;
-            const bool bump = mx2 > mr + 8.0f;           // also true while mr = -inf and a key is visible
-            const float mr_new = bump ? mx2 : mr;
-            float pv[64];
-            float sum = 0.f;
-            if (mr_new == -INFINITY) {
-#pragma unroll
-                for (int j = 0; j < 64; ++j) pv[j] = 0.f;
-            } else {
-#pragma unroll
-                for (int j = 0; j < 64; ++j) {
-                    pv[j] = ex2(fmaf(s[j], sl, -mr_new));
-                    sum += pv[j];
+                    for (int e = 0; e < 32; ++e) x[e] = w[c0 + e];
+                    tmem_st32(tmem + lane_off + C::TMEM_Q + half * W + c0, x);
                 }
+            } else {
+                uint32_t x[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) x[e] = w[e];
+                tmem_st16(tmem + lane_off + C::TMEM_Q + half * W, x);
             }
-            const float factor = bump ? ((mr == -INFINITY) ? 0.f : ex2(mr - mr_new)) : 1.f;
-            // P buffer and O are free once the previous PV has completed
-            if (i > 0) {
-                ok = wait_all(PV_DONE, (i - 1) & 1);
-                if (!ok) break;
+            tmem_st_wait();
+            tc_fence_before();
+            mbar_arrive(bar(Q_FULL));
+        };
+        if (more(t_begin, k_begin)) stage_q(t_begin);
+        int j = 0, seg = 0;
+        for (int t = t_begin, k = k_begin; more(t, k); ++t, k = 0, ++seg) {
+            const Tile T = decode_tile(p, t);
+            const AttnChar& ch = p.ch[T.b];
+            const int k1 = (t == t_end) ? k_end : T.nk;
+            const int n = k1 - k;
+            const bool full = (k == 0 && k1 == T.nk);
+            const bool has_next = more(t + 1, 0);
+            const int tok = T.tok0 + r / g;
+            const bool row_valid = tok < ch.M;
+            const int lim = ch.L_prev + min(tok, ch.M - 1) + 1;    // keys [0, lim) are visible
+            float mr = -INFINITY;                        // reference max, log2 units
+            float l = 0.f;                               // this half's share of the row sum
+            for (int i = 0; i < n; ++i, ++j) {
+                const int sb = j & 1;
+                wait_all(S_FULL + sb, (j >> 1) & 1, 0x31 + 256 * j);
                 tc_fence_after();
-                if (__any_sync(0xffffffffu, bump)) {
+                uint32_t sa[32];
+                tmem_ld32(tmem + lane_off + C::TMEM_S + sb * BN + 32 * half, sa);
+                tmem_ld_wait();
+                tc_fence_before();
+                mbar_arrive(bar(S_EMPTY + sb));
+                // the segment's last S has landed, so no MMA reads Q any more
+                if (i + 1 == n && has_next) stage_q(t + 1);
+                const int key0 = (k + i) * BN + 32 * half;
+                float s[32];
+#pragma unroll
+                for (int c = 0; c < 32; ++c) s[c] = __uint_as_float(sa[c]);
+                if (key0 + 32 > lim) {
+#pragma unroll
+                    for (int c = 0; c < 32; ++c)
+                        if (key0 + c >= lim) s[c] = -INFINITY;
+                }
+                float m16[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c) m16[c] = fmaxf(s[c], s[c + 16]);
+#pragma unroll
+                for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+                    for (int c = 0; c < w; ++c) m16[c] = fmaxf(m16[c], m16[c + w]);
+                const float pm = m16[0];
+                float* xs = xch + sb * 2 * BM;           // [half][row] of this tile
+                xs[half * BM + r] = pm;
+                named_bar_sync(pair_bar, 64);
+                const float mx2 = fmaxf(pm, xs[(1 - half) * BM + r]) * sl;
+                const bool bump = mx2 > mr + 8.0f;       // also true while mr = -inf and a key is visible
+                const float mr_new = bump ? mx2 : mr;
+                float pv[32];
+                float sum = 0.f;
+                if (mr_new == -INFINITY) {
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) pv[c] = 0.f;
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) pv[c] = ex2(fmaf(s[c], sl, -mr_new));
+                    float a16[16];
+#pragma unroll
+                    for (int c = 0; c < 16; ++c) a16[c] = pv[c] + pv[c + 16];
+#pragma unroll
+                    for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+                        for (int c = 0; c < w; ++c) a16[c] += a16[c + w];
+                    sum = a16[0];
+                }
+                const float factor = bump ? ((mr == -INFINITY) ? 0.f : ex2(mr - mr_new)) : 1.f;
+                // P buffer sb is free once PV_{j-2} has completed
+                if (j >= 2) wait_all(PV_DONE + sb, ((j >> 1) - 1) & 1, 0x32 + 256 * j);
+                if (i > 0 && __any_sync(0xffffffffu, bump)) {
+                    // rescale this half of the O row once PV_{j-1} has landed
+                    wait_all(PV_DONE + (sb ^ 1), ((j - 1) >> 1) & 1, 0x33 + 256 * j);
+                    tc_fence_after();
 #pragma unroll 1
-                    for (int c0 = 0; c0 < D; c0 += 32) {
+                    for (int c0 = half * C::HALF; c0 < (half + 1) * C::HALF; c0 += 32) {
                         uint32_t o[32];
                         tmem_ld32(tmem + lane_off + C::TMEM_O + c0, o);
                         tmem_ld_wait();
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * factor);
+                        for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * factor);
                         tmem_st32(tmem + lane_off + C::TMEM_O + c0, o);
                     }
                     tmem_st_wait();
                 }
-            }
-            l = l * factor + sum;
-            mr = mr_new;
-            // P row r: 64 bf16 = 8 chunks of 16 bytes, chunk index XOR (row & 7)
+                l = l * factor + sum;
+                mr = mr_new;
+                // 32 bf16 of row r = 16-byte chunks 4 half .. 4 half + 3, chunk index XOR (r & 7)
+                const uint32_t prow = sP + sb * C::P_BYTES + r * 128;
 #pragma unroll
-            for (int ch = 0; ch < 8; ++ch) {
-                uint32_t w[4];
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t w[4];
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    __nv_bfloat162 h2 = __floats2bfloat162_rn(pv[ch * 8 + 2 * e], pv[ch * 8 + 2 * e + 1]);
-                    w[e] = *reinterpret_cast<uint32_t*>(&h2);
+                    for (int e = 0; e < 4; ++e) {
+                        __nv_bfloat162 h2 = __floats2bfloat162_rn(pv[8 * q + 2 * e], pv[8 * q + 2 * e + 1]);
+                        w[e] = *reinterpret_cast<uint32_t*>(&h2);
+                    }
+                    st_shared_v4(prow + (((4 * half + q) ^ (r & 7)) << 4), w[0], w[1], w[2], w[3]);
                 }
-                st_shared_v4(sP + r * 128 + ((ch ^ (r & 7)) << 4), w[0], w[1], w[2], w[3]);
+                fence_proxy_async_smem();
+                tc_fence_before();
+                mbar_arrive(bar(P_FULL + sb));
             }
-            fence_proxy_async_smem();
-            tc_fence_before();
-            mbar_arrive(bar(P_FULL));
-        }
-        if (n > 0 && ok) ok = wait_all(O_FINAL, 0);
-        if (ok) {
+            // ---------------------------------------------------------------- epilogue of the segment
+            wait_all(O_FINAL, seg & 1, 0x34 + 256 * seg);
             tc_fence_after();
-            const int hq = kvh * g + (r % g);
-            const int64_t item_row = (int64_t)blockIdx.x * BM + r;
-            if (p.n_split == 1) {
-                // tcgen05.ld is warp-collective (.sync.aligned): every lane
-                // loads, and only lanes of real query rows store
-                const float inv = row_valid ? 1.f / l : 0.f;
-                __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + (row_valid ? tok : 0)) * p.Hq + hq) * D;
+            float* xl = xch + (j & 1) * 2 * BM;          // the exchange buffer the last tile did not use
+            xl[half * BM + r] = l;
+            named_bar_sync(pair_bar, 64);
+            const float lt = l + xl[(1 - half) * BM + r];
+            named_bar_sync(pair_bar, 64);                // the buffer is free for the next segment
+            const bool store = *abort_flag == 0;
+            const int hq = T.kvh * g + (r % g);
+            if (full) {
+                // tcgen05.ld is warp-collective: every lane loads, real rows store
+                const float inv = row_valid ? 1.f / lt : 0.f;
+                __nv_bfloat16* o = p.out + ((int64_t)(ch.tail_off + (row_valid ? tok : 0)) * p.Hq + hq) * D;
 #pragma unroll 1
-                for (int c0 = 0; c0 < D; c0 += 32) {
+                for (int c0 = half * C::HALF; c0 < (half + 1) * C::HALF; c0 += 32) {
                     uint32_t v[32];
                     tmem_ld32(tmem + lane_off + C::TMEM_O + c0, v);
                     tmem_ld_wait();
-                    if (row_valid) {
+                    if (row_valid && store) {
                         uint32_t w[16];
 #pragma unroll
                         for (int e = 0; e < 16; ++e) {
@@ -331,23 +451,38 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
                     }
                 }
             } else {
-                p.part_ml[item_row * 2 + 0] = mr;
-                p.part_ml[item_row * 2 + 1] = l;
-                if (n > 0) {
-                    float* o = p.part_o + item_row * D;
+                const int64_t prow = (int64_t)(2 * cta + (seg == 0 ? 0 : 1)) * BM + r;
+                if (half == 0 && store) {
+                    p.part_ml[prow * 2 + 0] = mr;
+                    p.part_ml[prow * 2 + 1] = lt;
+                }
+                // partial layout [slot][D / 32][row][32]: a warp stores 4 KB contiguously
+                const int64_t slot = 2 * cta + (seg == 0 ? 0 : 1);
 #pragma unroll 1
-                    for (int c0 = 0; c0 < D; c0 += 32) {
-                        uint32_t v[32];
-                        tmem_ld32(tmem + lane_off + C::TMEM_O + c0, v);
-                        tmem_ld_wait();
-                        uint4* dst = reinterpret_cast<uint4*>(o + c0);
+                for (int c0 = half * C::HALF; c0 < (half + 1) * C::HALF; c0 += 32) {
+                    uint32_t v[32];
+                    tmem_ld32(tmem + lane_off + C::TMEM_O + c0, v);
+                    tmem_ld_wait();
+                    if (store) {
+                        uint4* dst = reinterpret_cast<uint4*>(p.part_o + ((slot * (D / 32) + c0 / 32) * BM + r) * 32);
 #pragma unroll
                         for (int e = 0; e < 8; ++e) dst[e] = make_uint4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
                     }
                 }
             }
+            tc_fence_before();
+            mbar_arrive(bar(O_EMPTY));
         }
-        tc_fence_before();
+    }
+    tc_fence_before();
+    __syncthreads();
+    if ((warp == 0 || warp == kVWarp) && lane == 0 && *abort_flag) {
+        // copies still in flight land before the block releases its shared memory
+        volatile int never = 0;
+        const int full = warp == 0 ? K_FULL : V_FULL;
+        for (int s = 0; s < STAGES; ++s)
+            if (last_load[s] >= 0)
+                mbar_wait(bar(full + s), (last_load[s] / STAGES) & 1, &never, p.err, kErrWait, nullptr, 0, 100000000ull);
     }
     __syncthreads();
     if (warp == 1) {
@@ -366,13 +501,13 @@ void launch_tc(const AttnParams& p, cudaStream_t s) {
         cudaFuncSetAttribute(tail_attention_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         configured |= 1ull << (dev & 63);
     }
-    tail_attention_tc_kernel<D><<<p.n_items, kThreads, C::SMEM, s>>>(p);
+    tail_attention_tc_kernel<D><<<p.n_ctas, kThreads, C::SMEM, s>>>(p);
 }
 
 }  // namespace
 
 void launch_tail_attention(const AttnParams& p, cudaStream_t s) {
-    if (p.n_items <= 0) return;
+    if (p.n_ctas <= 0) return;
     switch (p.D) {
         case 64: launch_tc<64>(p, s); break;
         case 128: launch_tc<128>(p, s); break;
@@ -381,6 +516,8 @@ void launch_tail_attention(const AttnParams& p, cudaStream_t s) {
     }
 }
 
-int attention_rows_per_tile() { return BM; }
+// One block per SM: 320 threads of about 128 registers leave no room for a
+// second (and head_dim 256 needs all of TMEM and shared memory).
+int attention_ctas_per_sm(int) { return 1; }
 
 }  // namespace kvm
