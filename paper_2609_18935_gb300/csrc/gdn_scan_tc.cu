@@ -38,6 +38,7 @@ constexpr int kThreads = 256;
 constexpr int DVMAX = 128;       // d_v rows per scan block
 constexpr int DVP = 256;         // largest d_v the prep kernel stages
 constexpr int LSTRIDE = 68;      // fp32 row stride of the L scratch (conflict-free row vectors)
+constexpr int DSTRIDE = 20;      // fp32 row stride of the diagonal-block inverses
 
 // Workspace record of one (chunk, head):
 //   [W;Q'] hi | [W;Q'] lo   (128 x DK bf16 each, K-major 128-byte-swizzled image)
@@ -98,8 +99,14 @@ struct PrepCfg {
     static constexpr int OFF_L = OFF_V + V;                  // fp32 [64][LSTRIDE] L, then the A rows
     static constexpr int OFF_XG = OFF_L + 36864;             // X G hi, lo
     static constexpr int OFF_X = OFF_XG + 2 * TILE128;       // X hi, lo
-    static constexpr int OFF_BAR = OFF_X + 2 * TILE128;
+    static constexpr int OFF_D = OFF_X + 2 * TILE128;        // fp32 [64][DSTRIDE]: inverses of the diagonal blocks
+    static constexpr int OFF_BAR = OFF_D + 64 * DSTRIDE * 4;
     static constexpr int SMEM = OFF_BAR + 64 + 1024;
+    // record staging: [W;Q'] hi | lo over XG, X; U | A U over V, L
+    static constexpr int OFF_STAGE_WQ = OFF_XG;
+    static constexpr int OFF_STAGE_U = OFF_V;
+    static_assert(2 * 128 * DK * 2 <= 4 * TILE128, "[W;Q'] staging");
+    static_assert(128 * 128 * 4 <= V + 36864, "U | A U staging for d_v <= 128");
     static constexpr uint32_t T_D = 0;                       // KK / QK (64 cols)
     static constexpr uint32_t T_WU = 128;                    // [W | U] (DK + dv cols)
 };
@@ -145,6 +152,8 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
         tmem_alloc(smem_u32(tmem_slot), 512);
         tmem_relinquish();
     }
+    grid_dependency_wait();
+    grid_dependents_launch();
     // ---- loads (every global load issued before the shared stores)
     {
         constexpr int NKQ = 128 * (DK / 8) / kThreads;
@@ -169,8 +178,6 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
             const int i = tid + u * kThreads;
             const int rr = i / (DK / 8), c8 = (i % (DK / 8)) * 8;
             V4(oKQ + sw128_off16(rr, c8, 128)) = kq[u];
-            // the K image of the record (rows = tokens, 64-row regions)
-            if (rr < 64) *reinterpret_cast<uint4*>(rec + 2 * R::WQH + sw128_off16(rr, c8, 64)) = kq[u];
         }
 #pragma unroll
         for (int u = 0; u < NV; ++u) {
@@ -249,9 +256,30 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     }
     __syncthreads();
     // ---------------------------------------------------------------- X = [I; A] (I + L)^-1
-    // Two threads of one warp per row p (tid = 2p + h2): thread h2 owns the
-    // 8-column groups j8 = 16k + 8*h2; x (I + L) = b is solved right-looking,
-    // x_j -= x_i L[i][j] for j < i, i from 63 down, with x_i passed by shuffle.
+    // Each row x of X solves x (I + L) = b (b = e_p for p < 64, row p - 64 of
+    // A otherwise).  With I + L cut into 16 x 16 blocks (lower triangular by
+    // blocks, D_j the inverse of diagonal block j), the column blocks follow
+    // from the right: x_j = (b_j - sum_{i > j} x_i L_ij) D_j.  The D_j come
+    // first (thread t < 64 solves column t mod 16 of block t / 16).
+    float* Dm = reinterpret_cast<float*>(smem + G::OFF_D);
+    if (ok && tid < 64) {
+        const int kb = tid >> 4, c = tid & 15;
+        float d[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const float* li = Lm + (16 * kb + i) * LSTRIDE + 16 * kb;
+            float v = (i == c) ? 1.f : 0.f;
+#pragma unroll
+            for (int m = 0; m < i; ++m) v = fmaf(-li[m], d[m], v);
+            d[i] = v;
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) Dm[(16 * kb + i) * DSTRIDE + c] = d[i];
+    }
+    __syncthreads();
+    // Two threads per row p (tid = 2p + h2); thread h2 owns columns
+    // 16 k + 8 h2 .. + 7 of every block k.  Rows p < 64 are rows of the lower
+    // triangular T, zero right of column p: their warps skip those blocks.
     if (ok) {
         const int pr = tid >> 1, h2 = tid & 1;
         float xs[32];                                 // xs[8k + e] = x[16k + 8 h2 + e]
@@ -268,19 +296,46 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
                 xs[8 * k + 4] = b1.x; xs[8 * k + 5] = b1.y; xs[8 * k + 6] = b1.z; xs[8 * k + 7] = b1.w;
             }
         }
+        const int top = pr < 64 ? (pr >> 4) : 3;      // uniform per warp (16 rows of one block)
 #pragma unroll
-        for (int i = C - 1; i > 0; --i) {
-            const int owner = (i >> 3) & 1;
-            const float xi = __shfl_sync(0xffffffffu, xs[8 * (i >> 4) + (i & 7)], (lane & ~1) | owner);
+        for (int jb = 3; jb >= 0; --jb) {
+            if (jb > top) continue;
+            float y[16];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int j8 = 16 * k + 8 * h2;
-                if (j8 < i) {
-                    const float4 l0 = *reinterpret_cast<const float4*>(Lm + i * LSTRIDE + j8);
-                    const float4 l1 = *reinterpret_cast<const float4*>(Lm + i * LSTRIDE + j8 + 4);
+            for (int e = 0; e < 8; ++e) {
+                const float a = xs[8 * jb + e];
+                const float o = __shfl_xor_sync(0xffffffffu, a, 1);
+                y[8 * h2 + e] = a;
+                y[8 * (1 - h2) + e] = o;
+            }
+            float xb[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) xb[c] = 0.f;
+#pragma unroll
+            for (int m = 0; m < 16; ++m) {
+                const float4 d0 = *reinterpret_cast<const float4*>(Dm + (16 * jb + m) * DSTRIDE + 8 * h2);
+                const float4 d1 = *reinterpret_cast<const float4*>(Dm + (16 * jb + m) * DSTRIDE + 8 * h2 + 4);
+                const float dv8[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+#pragma unroll
+                for (int c = 0; c < 8; ++c) xb[c] = fmaf(y[m], dv8[c], xb[c]);
+            }
+            float xf[16];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                xs[8 * jb + c] = xb[c];
+                xf[8 * h2 + c] = xb[c];
+                xf[8 * (1 - h2) + c] = __shfl_xor_sync(0xffffffffu, xb[c], 1);
+            }
+#pragma unroll
+            for (int kb = 0; kb < jb; ++kb) {
+#pragma unroll
+                for (int m = 0; m < 16; ++m) {
+                    const float* lr = Lm + (16 * jb + m) * LSTRIDE + 16 * kb + 8 * h2;
+                    const float4 l0 = *reinterpret_cast<const float4*>(lr);
+                    const float4 l1 = *reinterpret_cast<const float4*>(lr + 4);
                     const float lv[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) xs[8 * k + e] = fmaf(-xi, lv[e], xs[8 * k + e]);   // L[i][j] = 0 for j >= i
+                    for (int c = 0; c < 8; ++c) xs[8 * kb + c] = fmaf(-xf[m], lv[c], xs[8 * kb + c]);
                 }
             }
         }
@@ -324,9 +379,12 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     }
     if (ok) ok = mma_wait();
     // ---------------------------------------------------------------- record: [W; Q'] image, U | A U
+    // Both are staged in shared memory in their record layout (the MMA
+    // operands they overwrite are consumed) and leave in bulk copies.
     if (ok) {
         const int t = row & 63;
         const float gt = Gs[t];
+        const uint32_t oWQ = G::OFF_STAGE_WQ;
         for (int cb = hf * (DK / 2); cb < (hf + 1) * (DK / 2); cb += 32) {
             uint32_t v[32];
             tmem_ld32(tmem + lane_off + G::T_WU + cb, v);
@@ -352,14 +410,14 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
             for (int j8 = 0; j8 < 32; j8 += 8) {
                 uint4 hi, lo;
                 split8(y + j8, hi, lo);
-                const int64_t off = sw128_off16(row, cb + j8, 128);
-                *reinterpret_cast<uint4*>(rec + off) = hi;
-                *reinterpret_cast<uint4*>(rec + R::WQH + off) = lo;
+                const uint32_t off = sw128_off16(row, cb + j8, 128);
+                V4(oWQ + off) = hi;
+                V4(oWQ + (uint32_t)R::WQH + off) = lo;
             }
         }
         const int dh = ((dv / 2) + 31) / 32 * 32;
         const int nc = dv / 4;                               // 16-byte chunks per row
-        float* uau = reinterpret_cast<float*>(rec + R::uau_off()) + (int64_t)row * dv;
+        const uint32_t urow = G::OFF_STAGE_U + (uint32_t)row * dv * 4;
         for (int rc = hf * dh; rc < min(dv, (hf + 1) * dh); rc += 32) {
             uint32_t v[32];
             tmem_ld32(tmem + lane_off + G::T_WU + DK + rc, v);
@@ -367,9 +425,19 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
 #pragma unroll
             for (int j4 = 0; j4 < 32; j4 += 4)
                 if (rc + j4 < dv)
-                    *reinterpret_cast<uint4*>(uau + 4 * (((rc + j4) / 4 + row) % nc)) =
-                        make_uint4(v[j4], v[j4 + 1], v[j4 + 2], v[j4 + 3]);
+                    V4(urow + 16u * (((rc + j4) / 4 + row) % nc)) = make_uint4(v[j4], v[j4 + 1], v[j4 + 2], v[j4 + 3]);
         }
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    if (ok && tid == 0) {
+        bulk_store(rec, sb + G::OFF_STAGE_WQ, 2 * (uint32_t)R::WQH);
+        // K image: rows 0..63 of each 64-column region of [K;Q]
+        for (int r = 0; r < DK / 64; ++r)
+            bulk_store(rec + 2 * R::WQH + r * (64 * 128), sb + oKQ + r * (128 * 128), 64 * 128);
+        bulk_store(rec + R::uau_off(), sb + G::OFF_STAGE_U, 128u * dv * 4u);
+        bulk_commit();
+        bulk_wait_all();
     }
     tc_fence_before();
     __syncthreads();
@@ -425,6 +493,8 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     const int h = blockIdx.y;
     const int b = blockIdx.z;
     const GdnChar ch = p.ch[b];
+    grid_dependency_wait();
+    grid_dependents_launch();
     if (ch.M <= 0) return;                           // uniform per block
     const int H = p.H, dv = p.dv;
     const int nch = (ch.M + C - 1) / C;
@@ -678,14 +748,14 @@ void configure_once(int smem) {
 template <int DK>
 void launch_prep_dk(const GdnParams& p, cudaStream_t s) {
     configure_once<gdn_prep_kernel<DK>>(PrepCfg<DK>::SMEM);
-    gdn_prep_kernel<DK><<<p.total_chunks * p.H, kThreads, PrepCfg<DK>::SMEM, s>>>(p);
+    launch_pdl(gdn_prep_kernel<DK>, dim3(p.total_chunks * p.H), dim3(kThreads), PrepCfg<DK>::SMEM, s, p);
 }
 
 template <int DK>
 void launch_scan_dk(const GdnParams& p, cudaStream_t s) {
     configure_once<gdn_scan_kernel<DK>>(ScanCfg<DK>::SMEM);
     dim3 grid(p.dv / p.dv_slice, p.H, p.n_chars);
-    gdn_scan_kernel<DK><<<grid, kThreads, ScanCfg<DK>::SMEM, s>>>(p);
+    launch_pdl(gdn_scan_kernel<DK>, grid, dim3(kThreads), ScanCfg<DK>::SMEM, s, p);
 }
 
 }  // namespace

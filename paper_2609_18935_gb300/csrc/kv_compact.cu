@@ -49,6 +49,8 @@ __device__ __forceinline__ int src_index(const int32_t* seg_start, const int32_t
 
 __global__ void __launch_bounds__(kCompactThreads)
 kv_compact_kernel(const __grid_constant__ CompactParams p) {
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int tid = threadIdx.x;
     // character of this block: last b with blk_off <= blockIdx.x
     int lo = 0, hi = p.n_chars - 1;
@@ -147,6 +149,8 @@ kv_compact_kernel(const __grid_constant__ CompactParams p) {
 }
 
 __global__ void gather_map_kernel(const __grid_constant__ GatherParams p) {
+    grid_dependency_wait();
+    grid_dependents_launch();
     for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < p.total; idx += gridDim.x * blockDim.x) {
         int lo = 0, hi = p.n_chars - 1;
         while (lo < hi) {
@@ -165,14 +169,14 @@ __global__ void gather_map_kernel(const __grid_constant__ GatherParams p) {
 
 void launch_kv_compact(const CompactParams& p, cudaStream_t s) {
     if (p.total_blocks <= 0) return;
-    kv_compact_kernel<<<p.total_blocks, kCompactThreads, 0, s>>>(p);
+    launch_pdl(kv_compact_kernel, dim3(p.total_blocks), dim3(kCompactThreads), 0, s, p);
 }
 
 void launch_gather_map(const GatherParams& p, cudaStream_t s) {
     if (p.total <= 0) return;
     int blocks = (p.total + 255) / 256;
     if (blocks > 4096) blocks = 4096;
-    gather_map_kernel<<<blocks, 256, 0, s>>>(p);
+    launch_pdl(gather_map_kernel, dim3(blocks), dim3(256), 0, s, p);
 }
 
 }  // namespace kvm

@@ -696,7 +696,17 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
     std::memset(&p, 0, sizeof p);
     p.n_chars = c->B;
     p.H = c->H; p.dk = c->dk; p.dv = c->dv;
-    p.dv_slice = c->dv;                 // one block carries all d_v rows of a head's state
+    // d_v rows of a head's state per scan block: split the rows (down to 32)
+    // until the (character, head, slice) blocks cover the SMs
+    {
+        int active = 0;
+        for (int b = 0; b < c->B; ++b) active += (tail_cu[b + 1] > tail_cu[b]);
+        int slices = 1;
+        while (c->dv / (2 * slices) >= 32 && c->dv % (2 * slices * 32) == 0 &&
+               (int64_t)active * c->H * slices < c->num_sms)
+            slices *= 2;
+        p.dv_slice = c->dv / slices;
+    }
     p.q = static_cast<const __nv_bfloat16*>(q);
     p.k = static_cast<const __nv_bfloat16*>(k);
     p.v = static_cast<const __nv_bfloat16*>(v);

@@ -9,6 +9,31 @@
 
 namespace kvm {
 
+// Programmatic dependent launch: every kernel of the library is launched so
+// that it may start while the previous kernel of the stream finishes.  A
+// kernel calls grid_dependency_wait() before its first global memory access
+// (it returns once the previous grid has completed and its writes are
+// visible), so stream order is kept; grid_dependents_launch() then lets the
+// next kernel's blocks be scheduled and run their prologue early.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dependents_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename Params>
+inline cudaError_t launch_pdl(void (*kernel)(Params), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              const Params& p) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, p);
+}
+
 constexpr int kMaxChars = 256;      // characters per context (per-round descriptors travel as kernel parameters)
 constexpr int kMaxSpans = 1024;     // deletion spans per round, all characters together
 constexpr int kMaxRotaryHalf = 128; // rotary_dim / 2

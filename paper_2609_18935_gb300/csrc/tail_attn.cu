@@ -43,6 +43,8 @@ __device__ __forceinline__ void rotate8(uint4& lo, uint4& hi, const float* cs, c
 }
 
 __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant__ AttnParams p) {
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int n = blockIdx.x;                 // packed tail token
     int lo = 0, hi = p.n_chars - 1;           // last b with tail_off <= n owns token n
     while (lo < hi) {
@@ -174,6 +176,8 @@ constexpr int kCombineRows = 4;
 __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant__ AttnParams p) {
     __shared__ float m_s[kCombineRows][kCombineMaxParts];
     __shared__ float l_s[kCombineRows][kCombineMaxParts];
+    grid_dependency_wait();
+    grid_dependents_launch();
     const int cb = p.split_cb[blockIdx.x];
     const int t = p.cta_tile[cb];
     const int c0 = cb - 1;
@@ -239,12 +243,12 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
 
 void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s) {
     if (total_tokens <= 0) return;
-    rope_append_kernel<<<total_tokens, 128, 0, s>>>(p);
+    launch_pdl(rope_append_kernel, dim3(total_tokens), dim3(128), 0, s, p);
 }
 
 void launch_attn_combine(const AttnParams& p, cudaStream_t s) {
     if (p.n_split_tiles <= 0) return;
-    attn_combine_kernel<<<dim3(p.n_split_tiles, kRows / kCombineRows), 256, 0, s>>>(p);
+    launch_pdl(attn_combine_kernel, dim3(p.n_split_tiles, kRows / kCombineRows), dim3(256), 0, s, p);
 }
 
 }  // namespace kvm

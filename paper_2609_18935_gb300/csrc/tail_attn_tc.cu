@@ -164,6 +164,8 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    grid_dependency_wait();
+    grid_dependents_launch();
 
     // copies issued by a producer lane (for the drain after an abort)
     int last_load[STAGES] = {-1, -1, -1};
@@ -501,7 +503,7 @@ void launch_tc(const AttnParams& p, cudaStream_t s) {
         cudaFuncSetAttribute(tail_attention_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         configured |= 1ull << (dev & 63);
     }
-    tail_attention_tc_kernel<D><<<p.n_ctas, kThreads, C::SMEM, s>>>(p);
+    launch_pdl(tail_attention_tc_kernel<D>, dim3(p.n_ctas), dim3(kThreads), C::SMEM, s, p);
 }
 
 }  // namespace
