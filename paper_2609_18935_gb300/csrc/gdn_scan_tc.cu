@@ -100,7 +100,8 @@ struct PrepCfg {
     static constexpr int OFF_XG = OFF_L + 36864;             // X G hi, lo
     static constexpr int OFF_X = OFF_XG + 2 * TILE128;       // X hi, lo
     static constexpr int OFF_D = OFF_X + 2 * TILE128;        // fp32 [64][DSTRIDE]: inverses of the diagonal blocks
-    static constexpr int OFF_BAR = OFF_D + 64 * DSTRIDE * 4;
+    static constexpr int OFF_Y = OFF_D + 64 * DSTRIDE * 4;   // fp32 [256][17]: one block of a row, per thread
+    static constexpr int OFF_BAR = OFF_Y + kThreads * 17 * 4;
     static constexpr int SMEM = OFF_BAR + 64 + 1024;
     // record staging: [W;Q'] hi | lo over XG, X; U | A U over V, L
     static constexpr int OFF_STAGE_WQ = OFF_XG;
@@ -214,8 +215,11 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     }
     uint32_t phase = 0;
     bool ok = true;
+    // the issuing thread waits for its MMAs and the block follows it at the
+    // barrier (waiting lanes of the issuer's warp would slow its issue)
     auto mma_wait = [&]() -> bool {
-        bool r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait, p.diag, 0x40);
+        bool r = true;
+        if (tid == 0) r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait, p.diag, 0x40);
         phase ^= 1;
         r = __syncthreads_and(r);
         tc_fence_after();
@@ -297,46 +301,58 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
             }
         }
         const int top = pr < 64 ? (pr >> 4) : 3;      // uniform per warp (16 rows of one block)
+        // the 16 values of the current block of this row (own 8 and the
+        // partner's 8) pass through this thread's slice of shared memory, so
+        // the 16-term loops need not be unrolled (the kernel runs once per
+        // SM; its code size costs instruction fetches)
+        float* yr = reinterpret_cast<float*>(smem + G::OFF_Y) + tid * 17;
 #pragma unroll
         for (int jb = 3; jb >= 0; --jb) {
             if (jb > top) continue;
-            float y[16];
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 const float a = xs[8 * jb + e];
                 const float o = __shfl_xor_sync(0xffffffffu, a, 1);
-                y[8 * h2 + e] = a;
-                y[8 * (1 - h2) + e] = o;
+                yr[8 * h2 + e] = a;
+                yr[8 * (1 - h2) + e] = o;
             }
             float xb[8];
 #pragma unroll
             for (int c = 0; c < 8; ++c) xb[c] = 0.f;
-#pragma unroll
+#pragma unroll 1
             for (int m = 0; m < 16; ++m) {
+                const float ym = yr[m];
                 const float4 d0 = *reinterpret_cast<const float4*>(Dm + (16 * jb + m) * DSTRIDE + 8 * h2);
                 const float4 d1 = *reinterpret_cast<const float4*>(Dm + (16 * jb + m) * DSTRIDE + 8 * h2 + 4);
-                const float dv8[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
-#pragma unroll
-                for (int c = 0; c < 8; ++c) xb[c] = fmaf(y[m], dv8[c], xb[c]);
+                xb[0] = fmaf(ym, d0.x, xb[0]); xb[1] = fmaf(ym, d0.y, xb[1]);
+                xb[2] = fmaf(ym, d0.z, xb[2]); xb[3] = fmaf(ym, d0.w, xb[3]);
+                xb[4] = fmaf(ym, d1.x, xb[4]); xb[5] = fmaf(ym, d1.y, xb[5]);
+                xb[6] = fmaf(ym, d1.z, xb[6]); xb[7] = fmaf(ym, d1.w, xb[7]);
             }
-            float xf[16];
 #pragma unroll
             for (int c = 0; c < 8; ++c) {
                 xs[8 * jb + c] = xb[c];
-                xf[8 * h2 + c] = xb[c];
-                xf[8 * (1 - h2) + c] = __shfl_xor_sync(0xffffffffu, xb[c], 1);
+                yr[8 * h2 + c] = xb[c];
+                yr[8 * (1 - h2) + c] = __shfl_xor_sync(0xffffffffu, xb[c], 1);
             }
 #pragma unroll
             for (int kb = 0; kb < jb; ++kb) {
+                float acc[8];
 #pragma unroll
+                for (int c = 0; c < 8; ++c) acc[c] = xs[8 * kb + c];
+#pragma unroll 1
                 for (int m = 0; m < 16; ++m) {
+                    const float xm = yr[m];
                     const float* lr = Lm + (16 * jb + m) * LSTRIDE + 16 * kb + 8 * h2;
                     const float4 l0 = *reinterpret_cast<const float4*>(lr);
                     const float4 l1 = *reinterpret_cast<const float4*>(lr + 4);
-                    const float lv[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
-#pragma unroll
-                    for (int c = 0; c < 8; ++c) xs[8 * kb + c] = fmaf(-xf[m], lv[c], xs[8 * kb + c]);
+                    acc[0] = fmaf(-xm, l0.x, acc[0]); acc[1] = fmaf(-xm, l0.y, acc[1]);
+                    acc[2] = fmaf(-xm, l0.z, acc[2]); acc[3] = fmaf(-xm, l0.w, acc[3]);
+                    acc[4] = fmaf(-xm, l1.x, acc[4]); acc[5] = fmaf(-xm, l1.y, acc[5]);
+                    acc[6] = fmaf(-xm, l1.z, acc[6]); acc[7] = fmaf(-xm, l1.w, acc[7]);
                 }
+#pragma unroll
+                for (int c = 0; c < 8; ++c) xs[8 * kb + c] = acc[c];
             }
         }
         // operands: X G (for W) and X (for U), K-major rows
@@ -437,7 +453,10 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
             bulk_store(rec + 2 * R::WQH + r * (64 * 128), sb + oKQ + r * (128 * 128), 64 * 128);
         bulk_store(rec + R::uau_off(), sb + G::OFF_STAGE_U, 128u * dv * 4u);
         bulk_commit();
-        bulk_wait_all();
+        // the sources must be read before the block's shared memory is
+        // released; the writes complete with the grid, before the scan
+        // (which waits on this grid) reads them
+        bulk_wait_read();
     }
     tc_fence_before();
     __syncthreads();
@@ -559,8 +578,11 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
 
     uint32_t phase = 0;
     bool ok = true;
+    // the issuing thread waits for its MMAs and the block follows it at the
+    // barrier (waiting lanes of the issuer's warp would slow its issue)
     auto mma_wait = [&]() -> bool {
-        bool r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait, p.diag, 0x50);
+        bool r = true;
+        if (tid == 0) r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait, p.diag, 0x50);
         phase ^= 1;
         r = __syncthreads_and(r);
         tc_fence_after();
