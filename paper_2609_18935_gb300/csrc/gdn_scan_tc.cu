@@ -96,12 +96,11 @@ struct PrepCfg {
     static constexpr int TILE128 = 128 * 64 * 2;             // 128 x 64 bf16 K-major tile
     static constexpr int OFF_KQ = 0;
     static constexpr int OFF_V = OFF_KQ + KQ;
-    static constexpr int OFF_L = OFF_V + V;                  // fp32 [64][LSTRIDE] L, then the A rows
+    static constexpr int OFF_L = OFF_V + V;                  // fp32 [64][LSTRIDE] L (and record staging)
     static constexpr int OFF_XG = OFF_L + 36864;             // X G hi, lo
     static constexpr int OFF_X = OFF_XG + 2 * TILE128;       // X hi, lo
     static constexpr int OFF_D = OFF_X + 2 * TILE128;        // fp32 [64][DSTRIDE]: inverses of the diagonal blocks
-    static constexpr int OFF_Y = OFF_D + 64 * DSTRIDE * 4;   // fp32 [256][17]: one block of a row, per thread
-    static constexpr int OFF_BAR = OFF_Y + kThreads * 17 * 4;
+    static constexpr int OFF_BAR = OFF_D + 64 * DSTRIDE * 4;
     static constexpr int SMEM = OFF_BAR + 64 + 1024;
     // record staging: [W;Q'] hi | lo over XG, X; U | A U over V, L
     static constexpr int OFF_STAGE_WQ = OFF_XG;
@@ -126,7 +125,6 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     uint64_t* bar = reinterpret_cast<uint64_t*>(smem + G::OFF_BAR);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + G::OFF_BAR + 8);
     const uint32_t mbar = smem_u32(bar);
-    float* Bm = Lm + 64 * LSTRIDE;                   // fp32 [64][LSTRIDE]: rows of A (right-hand sides)
     __shared__ float gs[C], bs[C], Gs[C], g2[C];
     __shared__ volatile int abort_flag;
 
@@ -238,6 +236,9 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     }
     ok = mma_wait();                                // also publishes Gs
     // ---------------------------------------------------------------- L (rows < 64), A (rows >= 64)
+    // L goes to shared memory in fp32 for the solve of T = (I + L)^-1; the
+    // rows of [I; A] go straight into the A operand of X = [I; A] T (bf16 hi |
+    // lo, K-major, over the XG tiles)
     if (ok) {
         // thread (row, hf) handles columns hf*32 .. hf*32+31 of TMEM row `row`
         uint32_t v[32];
@@ -245,26 +246,36 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
         tmem_ld_wait();
         const int t = row & 63;
         const float gt2 = g2[t];
-        float* dst = (row < 64 ? Lm : Bm) + t * LSTRIDE + hf * 32;
+        float y[32];
 #pragma unroll
-        for (int j4 = 0; j4 < 32; j4 += 4) {
-            float y[4];
+        for (int c = 0; c < 32; ++c) {
+            const int j = hf * 32 + c;
+            const bool keep = (row < 64) ? (j < t) : (j <= t);
+            y[c] = (keep && t < n) ? ex2(gt2 - g2[j]) * bs[j] * __uint_as_float(v[c]) : 0.f;
+        }
+        if (row < 64) {
+            float* dst = Lm + t * LSTRIDE + hf * 32;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int j = hf * 32 + j4 + e;
-                const bool keep = (row < 64) ? (j < t) : (j <= t);
-                y[e] = (keep && t < n) ? ex2(gt2 - g2[j]) * bs[j] * __uint_as_float(v[j4 + e]) : 0.f;
-            }
-            *reinterpret_cast<float4*>(dst + j4) = make_float4(y[0], y[1], y[2], y[3]);
+            for (int j4 = 0; j4 < 32; j4 += 4) *reinterpret_cast<float4*>(dst + j4) = make_float4(y[j4], y[j4 + 1], y[j4 + 2], y[j4 + 3]);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) y[c] = (hf * 32 + c == row) ? 1.f : 0.f;     // row of I
+        }
+#pragma unroll
+        for (int j8 = 0; j8 < 32; j8 += 8) {
+            uint4 hi, lo;
+            split8(y + j8, hi, lo);
+            const uint32_t off = sw128_off16(row, hf * 32 + j8, 128);
+            V4(oXG + off) = hi;
+            V4(oXG + T128 + off) = lo;
         }
     }
     __syncthreads();
-    // ---------------------------------------------------------------- X = [I; A] (I + L)^-1
-    // Each row x of X solves x (I + L) = b (b = e_p for p < 64, row p - 64 of
-    // A otherwise).  With I + L cut into 16 x 16 blocks (lower triangular by
-    // blocks, D_j the inverse of diagonal block j), the column blocks follow
-    // from the right: x_j = (b_j - sum_{i > j} x_i L_ij) D_j.  The D_j come
-    // first (thread t < 64 solves column t mod 16 of block t / 16).
+    // ---------------------------------------------------------------- T = (I + L)^-1
+    // With I + L cut into 16 x 16 blocks (lower triangular by blocks, D_j the
+    // inverse of diagonal block j), row p of T solves x (I + L) = e_p column
+    // block by column block from the right: x_j = (b_j - sum_{i > j} x_i L_ij) D_j,
+    // zero right of column p.  The D_j come first (thread t < 64 solves
+    // column t mod 16 of block t / 16).
     float* Dm = reinterpret_cast<float*>(smem + G::OFF_D);
     if (ok && tid < 64) {
         const int kb = tid >> 4, c = tid & 15;
@@ -281,93 +292,117 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
         for (int i = 0; i < 16; ++i) Dm[(16 * kb + i) * DSTRIDE + c] = d[i];
     }
     __syncthreads();
-    // Two threads per row p (tid = 2p + h2); thread h2 owns columns
-    // 16 k + 8 h2 .. + 7 of every block k.  Rows p < 64 are rows of the lower
-    // triangular T, zero right of column p: their warps skip those blocks.
+    // Four threads per row p (tid = 4p + q); thread q owns columns
+    // 16 k + 4 q .. + 3 of every block k; warps of rows in block top skip the
+    // blocks right of it.  T leaves as the B operand (MN-major, rows = the
+    // contraction index) of X = [I; A] T, bf16 hi | lo over the X tiles.
     if (ok) {
-        const int pr = tid >> 1, h2 = tid & 1;
-        float xs[32];                                 // xs[8k + e] = x[16k + 8 h2 + e]
+        const int pr = tid >> 2, q = tid & 3;
+        float xs[16];                                 // xs[4k + e] = x[16k + 4q + e]
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int j8 = 16 * k + 8 * h2;
-            if (pr < 64) {
+        for (int k = 0; k < 4; ++k)
 #pragma unroll
-                for (int e = 0; e < 8; ++e) xs[8 * k + e] = (j8 + e == pr) ? 1.f : 0.f;
-            } else {
-                const float4 b0 = *reinterpret_cast<const float4*>(Bm + (pr - 64) * LSTRIDE + j8);
-                const float4 b1 = *reinterpret_cast<const float4*>(Bm + (pr - 64) * LSTRIDE + j8 + 4);
-                xs[8 * k + 0] = b0.x; xs[8 * k + 1] = b0.y; xs[8 * k + 2] = b0.z; xs[8 * k + 3] = b0.w;
-                xs[8 * k + 4] = b1.x; xs[8 * k + 5] = b1.y; xs[8 * k + 6] = b1.z; xs[8 * k + 7] = b1.w;
-            }
-        }
-        const int top = pr < 64 ? (pr >> 4) : 3;      // uniform per warp (16 rows of one block)
-        // the 16 values of the current block of this row (own 8 and the
-        // partner's 8) pass through this thread's slice of shared memory, so
-        // the 16-term loops need not be unrolled (the kernel runs once per
-        // SM; its code size costs instruction fetches)
-        float* yr = reinterpret_cast<float*>(smem + G::OFF_Y) + tid * 17;
+            for (int e = 0; e < 4; ++e) xs[4 * k + e] = (16 * k + 4 * q + e == pr) ? 1.f : 0.f;
+        const int top = pr >> 4;                      // uniform per warp (8 rows of one block)
 #pragma unroll
         for (int jb = 3; jb >= 0; --jb) {
             if (jb > top) continue;
+            // yv[o][e] = current x[16 jb + 4 (q ^ o) + e]
+            float yv[4][4];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const float a = xs[8 * jb + e];
-                const float o = __shfl_xor_sync(0xffffffffu, a, 1);
-                yr[8 * h2 + e] = a;
-                yr[8 * (1 - h2) + e] = o;
+            for (int e = 0; e < 4; ++e) {
+                const float a = xs[4 * jb + e];
+                yv[0][e] = a;
+                yv[1][e] = __shfl_xor_sync(0xffffffffu, a, 1);
+                yv[2][e] = __shfl_xor_sync(0xffffffffu, a, 2);
+                yv[3][e] = __shfl_xor_sync(0xffffffffu, a, 3);
             }
-            float xb[8];
+            float xb[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int c = 0; c < 8; ++c) xb[c] = 0.f;
-#pragma unroll 1
-            for (int m = 0; m < 16; ++m) {
-                const float ym = yr[m];
-                const float4 d0 = *reinterpret_cast<const float4*>(Dm + (16 * jb + m) * DSTRIDE + 8 * h2);
-                const float4 d1 = *reinterpret_cast<const float4*>(Dm + (16 * jb + m) * DSTRIDE + 8 * h2 + 4);
-                xb[0] = fmaf(ym, d0.x, xb[0]); xb[1] = fmaf(ym, d0.y, xb[1]);
-                xb[2] = fmaf(ym, d0.z, xb[2]); xb[3] = fmaf(ym, d0.w, xb[3]);
-                xb[4] = fmaf(ym, d1.x, xb[4]); xb[5] = fmaf(ym, d1.y, xb[5]);
-                xb[6] = fmaf(ym, d1.z, xb[6]); xb[7] = fmaf(ym, d1.w, xb[7]);
-            }
+            for (int o = 0; o < 4; ++o)
 #pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                xs[8 * jb + c] = xb[c];
-                yr[8 * h2 + c] = xb[c];
-                yr[8 * (1 - h2) + c] = __shfl_xor_sync(0xffffffffu, xb[c], 1);
-            }
-#pragma unroll
-            for (int kb = 0; kb < jb; ++kb) {
-                float acc[8];
-#pragma unroll
-                for (int c = 0; c < 8; ++c) acc[c] = xs[8 * kb + c];
-#pragma unroll 1
-                for (int m = 0; m < 16; ++m) {
-                    const float xm = yr[m];
-                    const float* lr = Lm + (16 * jb + m) * LSTRIDE + 16 * kb + 8 * h2;
-                    const float4 l0 = *reinterpret_cast<const float4*>(lr);
-                    const float4 l1 = *reinterpret_cast<const float4*>(lr + 4);
-                    acc[0] = fmaf(-xm, l0.x, acc[0]); acc[1] = fmaf(-xm, l0.y, acc[1]);
-                    acc[2] = fmaf(-xm, l0.z, acc[2]); acc[3] = fmaf(-xm, l0.w, acc[3]);
-                    acc[4] = fmaf(-xm, l1.x, acc[4]); acc[5] = fmaf(-xm, l1.y, acc[5]);
-                    acc[6] = fmaf(-xm, l1.z, acc[6]); acc[7] = fmaf(-xm, l1.w, acc[7]);
+                for (int e = 0; e < 4; ++e) {
+                    const float4 d4 = *reinterpret_cast<const float4*>(Dm + (16 * jb + 4 * (q ^ o) + e) * DSTRIDE + 4 * q);
+                    xb[0] = fmaf(yv[o][e], d4.x, xb[0]); xb[1] = fmaf(yv[o][e], d4.y, xb[1]);
+                    xb[2] = fmaf(yv[o][e], d4.z, xb[2]); xb[3] = fmaf(yv[o][e], d4.w, xb[3]);
                 }
+            float xv[4][4];
 #pragma unroll
-                for (int c = 0; c < 8; ++c) xs[8 * kb + c] = acc[c];
+            for (int c = 0; c < 4; ++c) {
+                xs[4 * jb + c] = xb[c];
+                xv[0][c] = xb[c];
+                xv[1][c] = __shfl_xor_sync(0xffffffffu, xb[c], 1);
+                xv[2][c] = __shfl_xor_sync(0xffffffffu, xb[c], 2);
+                xv[3][c] = __shfl_xor_sync(0xffffffffu, xb[c], 3);
             }
+#pragma unroll
+            for (int kb = 0; kb < jb; ++kb)
+#pragma unroll
+                for (int o = 0; o < 4; ++o)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float4 l4 = *reinterpret_cast<const float4*>(
+                            Lm + (16 * jb + 4 * (q ^ o) + e) * LSTRIDE + 16 * kb + 4 * q);
+                        xs[4 * kb + 0] = fmaf(-xv[o][e], l4.x, xs[4 * kb + 0]);
+                        xs[4 * kb + 1] = fmaf(-xv[o][e], l4.y, xs[4 * kb + 1]);
+                        xs[4 * kb + 2] = fmaf(-xv[o][e], l4.z, xs[4 * kb + 2]);
+                        xs[4 * kb + 3] = fmaf(-xv[o][e], l4.w, xs[4 * kb + 3]);
+                    }
         }
-        // operands: X G (for W) and X (for U), K-major rows
+        // T row pr, columns 16 k + 4 q .. + 3: 8 bytes of each of hi and lo
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            const int j8 = 16 * k + 8 * h2;
-            float xg[8];
+            float hi4[4], lo4[4];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) xg[e] = xs[8 * k + e] * Gs[j8 + e];
+            for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat16 h = __float2bfloat16_rn(xs[4 * k + e]);
+                hi4[e] = __bfloat162float(h);
+                lo4[e] = xs[4 * k + e] - hi4[e];
+            }
+            const uint32_t off = sw128_off16(pr, 16 * k + 4 * q, 64);
+            *reinterpret_cast<uint2*>(smem + oX + off) = make_uint2(pack_bf16x2(hi4[0], hi4[1]), pack_bf16x2(hi4[2], hi4[3]));
+            *reinterpret_cast<uint2*>(smem + oX + 64 * 128 + off) = make_uint2(pack_bf16x2(lo4[0], lo4[1]), pack_bf16x2(lo4[2], lo4[3]));
+        }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    // ---------------------------------------------------------------- X = [I; A] T on the tensor cores
+    if (ok && tid == 0) {
+        tc_fence_after();
+        const uint32_t id_x = idesc_bf16_f32(128, C, true);          // B = T, MN-major
+#pragma unroll
+        for (int ks = 0; ks < C / 16; ++ks) {
+            const uint64_t a_hi = smem_desc_sw128(sb + oXG + ks * 32, 16, 1024);
+            const uint64_t a_lo = smem_desc_sw128(sb + oXG + T128 + ks * 32, 16, 1024);
+            const uint64_t b_hi = smem_desc_sw128(sb + oX + ks * 16 * 128, C * 128, 1024);
+            const uint64_t b_lo = smem_desc_sw128(sb + oX + 64 * 128 + ks * 16 * 128, C * 128, 1024);
+            mma_bf16(tmem + G::T_D, a_hi, b_hi, id_x, ks > 0);
+            mma_bf16(tmem + G::T_D, a_hi, b_lo, id_x, 1u);
+            mma_bf16(tmem + G::T_D, a_lo, b_hi, id_x, 1u);
+        }
+        mma_commit(mbar);
+    }
+    if (ok) ok = mma_wait();
+    // operands: X G (for W) and X (for U), K-major rows, from TMEM
+    if (ok) {
+        uint32_t v[32];
+        tmem_ld32(tmem + lane_off + G::T_D + hf * 32, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int j8 = 0; j8 < 32; j8 += 8) {
+            float xr[8], xg[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                xr[e] = __uint_as_float(v[j8 + e]);
+                xg[e] = xr[e] * Gs[hf * 32 + j8 + e];
+            }
             uint4 hi, lo;
+            const uint32_t off = sw128_off16(row, hf * 32 + j8, 128);
             split8(xg, hi, lo);
-            const uint32_t off = sw128_off16(pr, j8, 128);
             V4(oXG + off) = hi;
             V4(oXG + T128 + off) = lo;
-            split8(xs + 8 * k, hi, lo);
+            split8(xr, hi, lo);
             V4(oX + off) = hi;
             V4(oX + T128 + off) = lo;
         }
