@@ -208,8 +208,39 @@ def blas_threads() -> int:
     return os.cpu_count() or 1
 
 
+# ----------------------------------------------------------------------------
+# ranks (one process per GPU; replicas maintain different characters)
+# ----------------------------------------------------------------------------
+def dist_env():
+    """(rank, world size, local rank) from the launcher's environment."""
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def replica_seed(rank: int) -> int:
+    """Seed base of a rank's characters: every rank maintains its own."""
+    return 7919 * (rank + 1)
+
+
+def max_over_ranks(x: float, world: int, device="cpu") -> float:
+    """The job's time is the slowest rank's (all_reduce MAX); x itself on one rank."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, tokens_per_rank: float, ms: float) -> float:
+    """Whole-job tail tokens/s: every rank processes tokens_per_rank in the
+    job's time (the slowest rank's) of ms milliseconds."""
+    return world * tokens_per_rank / (ms / 1e3)
+
+
 def run_reference(args):
-    rank = int(os.environ.get("RANK", "0"))
+    rank, _, _ = dist_env()
     if rank != 0:
         return
     w = W.make_workload(args.workload)
@@ -242,9 +273,7 @@ def run_kvm(args):
     import torch.distributed as dist
     from paper_2609_18935_gb300 import build_lib, kvm
 
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    rank, world, local = dist_env()
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
@@ -262,7 +291,7 @@ def run_kvm(args):
     caps = w.capacity()
     mk = lambda max_tail: kvm.Context(s.layer_kind, s.n_q_heads, s.n_kv_heads, s.head_dim, s.rotary_dim,
                                       s.rope_theta, s.n_gdn_heads, s.d_k, s.d_v, caps, max_tail)
-    seed_base = 7919 * (rank + 1)        # each rank maintains its own characters
+    seed_base = replica_seed(rank)
 
     # ---- prefix root: a GPU refill of the prefix (no removals, tail = prefix)
     N = list(w.prefix_len)
@@ -359,11 +388,7 @@ def run_kvm(args):
         work.profile_read(0, reset=True)
         work.profile_enable(False)
         launches = work.launch_count() - launches0
-        total_ms = float(sum(ms))
-        if world > 1:
-            t = torch.tensor([total_ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            total_ms = float(t.item())
+        total_ms = max_over_ranks(float(sum(ms)), world, device="cuda")
         return total_ms, [r for _, _, r in evs], kernels, launches, (t0, t1)
 
     clocks = ClockSampler(local)
@@ -377,8 +402,8 @@ def run_kvm(args):
     clocks.stop()
 
     toks_rank = sum(sum(rounds[r]["tails"]) for r in rids)
-    value = world * toks_rank / (total_ms / 1e3)
-    e2e_value = world * sum(sum(rounds[r]["tails"]) for r in e2e_rids) / (e2e_ms / 1e3)
+    value = job_throughput(world, toks_rank, total_ms)
+    e2e_value = job_throughput(world, sum(sum(rounds[r]["tails"]) for r in e2e_rids), e2e_ms)
     hbm, tc_burst, tc_sust, peak_src = load_peaks()
     n_attn, n_gdn = len(s.attn_layers), len(s.gdn_layers)
     # algorithmic work of every kernel family over the timed steps
