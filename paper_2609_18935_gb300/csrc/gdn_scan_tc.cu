@@ -547,9 +547,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     const int h = blockIdx.y;
     const int b = blockIdx.z;
     const GdnChar ch = p.ch[b];
-    grid_dependency_wait();
-    grid_dependents_launch();
-    if (ch.M <= 0) return;                           // uniform per block
+    if (ch.M <= 0) return;                           // uniform per block; touches no memory
     const int H = p.H, dv = p.dv;
     const int nch = (ch.M + C - 1) / C;
     const int nc = dv / 4;                           // 16-byte chunks of a U | A U row
@@ -566,13 +564,6 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         mbar_init(bar_k, 1);
         mbar_init(bar_u, 1);
         fence_mbar_init();
-        // chunk 0's records
-        mbar_arrive_expect_tx(bar_wq, G::WQ);
-        bulk_load(sb + G::OFF_WQ, rec_of(0), G::WQ, bar_wq);
-        mbar_arrive_expect_tx(bar_k, G::KI);
-        bulk_load(sb + G::OFF_K, rec_of(0) + G::WQ, G::KI, bar_k);
-        mbar_arrive_expect_tx(bar_u, ubytes);
-        bulk_load(sb + G::OFF_U, rec_of(0) + R::uau_off(), ubytes, bar_u);
     }
     if (warp == 0) {
         tmem_alloc(smem_u32(tmem_slot), 256);
@@ -610,6 +601,19 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         if (row < DK) write_s_row(row, rc, sx);
     }
     tmem_st_wait();
+    // The state slice comes from an earlier round (or kvm_set_state), which
+    // completed before the prep kernel this launch follows had started, so
+    // it is staged before waiting for that kernel; its records are not.
+    grid_dependency_wait();
+    grid_dependents_launch();
+    if (tid == 0) {
+        mbar_arrive_expect_tx(bar_wq, G::WQ);
+        bulk_load(sb + G::OFF_WQ, rec_of(0), G::WQ, bar_wq);
+        mbar_arrive_expect_tx(bar_k, G::KI);
+        bulk_load(sb + G::OFF_K, rec_of(0) + G::WQ, G::KI, bar_k);
+        mbar_arrive_expect_tx(bar_u, ubytes);
+        bulk_load(sb + G::OFF_U, rec_of(0) + R::uau_off(), ubytes, bar_u);
+    }
 
     uint32_t phase = 0;
     bool ok = true;

@@ -164,7 +164,12 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    grid_dependency_wait();
+    // The kernel before this one (rope_append) writes the tail's keys and
+    // values and the rotated q; the surviving rows [0, L') were written
+    // earlier (by kv_compact, complete before rope_append began).  So the
+    // producers stream survivor tiles at once and wait for the previous grid
+    // only before a tile that reaches the tail; the softmax warps wait before
+    // staging Q.  The issuers touch no global memory.
     grid_dependents_launch();
 
     // copies issued by a producer lane (for the drain after an abort)
@@ -178,7 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
             const uint32_t ring = is_k ? sK : sV;
             const int full = is_k ? K_FULL : V_FULL, empty = is_k ? K_EMPTY : V_EMPTY;
             prefetch_tmap(map);
-            bool ok = true;
+            bool ok = true, waited = false;
             int j = 0;
             for (int t = t_begin, k = k_begin; ok && more(t, k); ++t, k = 0) {
                 const Tile T = decode_tile(p, t);
@@ -186,6 +191,10 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
                 const int k1 = (t == t_end) ? k_end : T.nk;
                 const int key_row0 = (p.attn_layer * p.Hkv + T.kvh) * (int)p.slab_rows + ch.cap_off;
                 for (int kt = k; kt < k1; ++kt, ++j) {
+                    if (!waited && (kt + 1) * BN > ch.L_prev) {    // the tile reaches the tail
+                        grid_dependency_wait();
+                        waited = true;
+                    }
                     const int st = j % STAGES;
                     if (j >= STAGES)
                         ok = mbar_wait(bar(empty + st), (j / STAGES - 1) & 1, abort_flag, p.err, kErrWait, p.diag,
@@ -290,6 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
         // Q tile of query tile t into TMEM: this thread's half of row r (D / 2
         // bf16 = D / 4 columns); rows past the character's tail are zero
         auto stage_q = [&](int t) {
+            grid_dependency_wait();                        // q_rot comes from the previous grid
             const Tile T = decode_tile(p, t);
             const AttnChar& ch = p.ch[T.b];
             const int tok = T.tok0 + r / g;
