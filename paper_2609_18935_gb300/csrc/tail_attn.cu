@@ -162,20 +162,15 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
     if (threadIdx.x == 0) p.pos[slot] = (int32_t)pos;
 }
 
-// grid (n_split_tiles, kRows / 4): block (x, y) merges rows 4y .. 4y + 3 of
-// the x-th query tile that several attention blocks share.  Block cb =
-// split_cb[x] is the first to start inside the tile, so its partials are in
-// the slots of blocks c0 = cb - 1 .. c1 (the last block that starts inside the
-// tile): c0's last segment (slot 2 c0 + 1, or 2 c0 when the tile is also c0's
-// first segment) and the first segments 2 c of the others.  The rows' (max,
-// sum) pairs are loaded together into shared memory, the weights
-// 2^(m_q - max) / sum formed once per row, and each thread then owns four
-// columns of one row and reads every partial's piece with independent loads.
-constexpr int kCombineMaxParts = kMaxAttnCtas + 1;
-constexpr int kCombineRows = 4;
+// grid (n_split_tiles, kRows * D / 4 / 256): the x-th query tile that several
+// attention blocks share.  Block cb = split_cb[x] is the first to start
+// inside the tile, so its partials are in the slots of blocks c0 = cb - 1 ..
+// c1 (the last block that starts inside the tile): c0's last segment (slot
+// 2 c0 + 1, or 2 c0 when the tile is also c0's first segment) and the first
+// segments 2 c of the others.  A thread owns four columns of one row and
+// merges the partials online, eight at a time, each batch's (max, sum) pairs
+// and O pieces loaded together.
 __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant__ AttnParams p) {
-    __shared__ float m_s[kCombineRows][kCombineMaxParts];
-    __shared__ float l_s[kCombineRows][kCombineMaxParts];
     grid_dependency_wait();
     grid_dependents_launch();
     const int cb = p.split_cb[blockIdx.x];
@@ -186,28 +181,6 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
     const int slot0 = (p.cta_tile[c0] == t) ? 2 * c0 : 2 * c0 + 1;
     const int n_parts = c1 - c0 + 1;
     auto slot_of = [&](int q) -> int64_t { return q == 0 ? slot0 : 2 * (c0 + q); };
-    const int row0 = blockIdx.y * kCombineRows;
-    for (int e = threadIdx.x; e < kCombineRows * n_parts; e += blockDim.x) {
-        const int rr = e / n_parts, q = e % n_parts;
-        const float2 ml = *reinterpret_cast<const float2*>(p.part_ml + (slot_of(q) * kRows + row0 + rr) * 2);
-        m_s[rr][q] = ml.x;
-        l_s[rr][q] = ml.y;
-    }
-    __syncthreads();
-    if (threadIdx.x < kCombineRows) {
-        const int rr = threadIdx.x;
-        float mx = -INFINITY;
-        for (int q = 0; q < n_parts; ++q) mx = fmaxf(mx, m_s[rr][q]);
-        float den = 0.f;
-        for (int q = 0; q < n_parts; ++q) {
-            const float w = (m_s[rr][q] == -INFINITY) ? 0.f : exp2f(m_s[rr][q] - mx);
-            m_s[rr][q] = w;                                        // the weight replaces the max
-            den += w * l_s[rr][q];
-        }
-        const float inv = den > 0.f ? 1.f / den : 0.f;
-        for (int q = 0; q < n_parts; ++q) m_s[rr][q] *= inv;
-    }
-    __syncthreads();
 
     int lo = 0, hi = p.n_chars - 1;                                // last b with tile_off <= t
     while (lo < hi) {
@@ -219,24 +192,50 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
     const int kvh = local / c.n_qtiles, qt = local % c.n_qtiles;
     const int D = p.D;
     const int groups = D / 32;                                     // 32-column groups
-    for (int idx = threadIdx.x; idx < kCombineRows * groups * 8; idx += blockDim.x) {
-        const int q4 = idx & 7;                                    // 4-column piece of the group
-        const int cg = (idx >> 3) % groups;
-        const int rr = (idx >> 3) / groups;
-        const int r = row0 + rr;
-        const int tok = qt * p.tok_per_tile + r / p.g;
-        if (tok >= c.M) continue;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-        for (int q = 0; q < n_parts; ++q) {
-            const float w = m_s[rr][q];
-            const float4 x = *reinterpret_cast<const float4*>(p.part_o + ((slot_of(q) * groups + cg) * kRows + r) * 32 + q4 * 4);
-            acc.x += w * x.x; acc.y += w * x.y; acc.z += w * x.z; acc.w += w * x.w;
+    const int item = blockIdx.y * blockDim.x + threadIdx.x;        // (row, 4-column piece)
+    const int r = item / (D / 4);
+    if (r >= kRows) return;
+    const int piece = item % (D / 4);
+    const int cg = piece >> 3, q4 = piece & 7;
+    const int tok = qt * p.tok_per_tile + r / p.g;
+    if (tok >= c.M) return;
+    constexpr int kBatch = 8;
+    float mx = -INFINITY, den = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int q0 = 0; q0 < n_parts; q0 += kBatch) {
+        float2 ml[kBatch];
+        float4 x[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            if (q0 + u < n_parts) {
+                const int64_t slot = slot_of(q0 + u);
+                ml[u] = *reinterpret_cast<const float2*>(p.part_ml + (slot * kRows + r) * 2);
+                x[u] = *reinterpret_cast<const float4*>(p.part_o + ((slot * groups + cg) * kRows + r) * 32 + q4 * 4);
+            } else {
+                ml[u] = make_float2(-INFINITY, 0.f);
+            }
         }
-        const int hq = kvh * p.g + (r % p.g);
-        __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + hq) * D + cg * 32 + q4 * 4;
-        *reinterpret_cast<uint2*>(o) = make_uint2(f2_to_bf2(acc.x, acc.y), f2_to_bf2(acc.z, acc.w));
+        float bm = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) bm = fmaxf(bm, ml[u].x);
+        const float nmx = fmaxf(mx, bm);
+        if (nmx == -INFINITY) continue;
+        const float sc = (mx == -INFINITY) ? 0.f : exp2f(mx - nmx);
+        den *= sc;
+        acc.x *= sc; acc.y *= sc; acc.z *= sc; acc.w *= sc;
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            if (ml[u].x == -INFINITY) continue;
+            const float w = exp2f(ml[u].x - nmx);
+            den += w * ml[u].y;
+            acc.x += w * x[u].x; acc.y += w * x[u].y; acc.z += w * x[u].z; acc.w += w * x[u].w;
+        }
+        mx = nmx;
     }
+    const float inv = den > 0.f ? 1.f / den : 0.f;
+    const int hq = kvh * p.g + (r % p.g);
+    __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + hq) * D + cg * 32 + q4 * 4;
+    *reinterpret_cast<uint2*>(o) = make_uint2(f2_to_bf2(acc.x * inv, acc.y * inv), f2_to_bf2(acc.z * inv, acc.w * inv));
 }
 
 }  // namespace
@@ -248,7 +247,7 @@ void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s) {
 
 void launch_attn_combine(const AttnParams& p, cudaStream_t s) {
     if (p.n_split_tiles <= 0) return;
-    launch_pdl(attn_combine_kernel, dim3(p.n_split_tiles, kRows / kCombineRows), dim3(256), 0, s, p);
+    launch_pdl(attn_combine_kernel, dim3(p.n_split_tiles, (kRows * (p.D / 4) + 255) / 256), dim3(256), 0, s, p);
 }
 
 }  // namespace kvm
