@@ -115,18 +115,28 @@ kv_compact_kernel(const __grid_constant__ CompactParams p) {
     }
     __threadfence();
     __syncthreads();
-    if (tid == 0) {
-        st_release(p.flags + flag_base + chunk, p.epoch);
-        // wait for earlier chunks whose sources reach into [d0, d1)
+    if (tid == 0) st_release(p.flags + (int64_t)(flag_base + chunk) * p.flag_stride, p.epoch);
+    if (tid < 32) {
+        // earlier chunks whose sources reach into [d0, d1) are e_min .. chunk - 1
+        // (their last sources are ordered); the lanes of warp 0 wait on their
+        // flags together, one flag each, so the waits cost one round trip
+        int e_min = chunk;
         for (int e = chunk - 1; e >= 0; --e) {
             const int last_dst = min(c.first + (e + 1) * rows, c.L_new) - 1;
             if (src_index(seg_start, seg_shift, c.n_seg, last_dst) < d0) break;
+            e_min = e;
+        }
+        bool fail = false;
+        for (int e = e_min + tid; e < chunk && !fail; e += 32) {
             int it = 0;
-            while (ld_acquire(p.flags + flag_base + e) != p.epoch) {
-                if (++it > kWaitLimit) { atomicOr(p.err, kErrWait); s_abort = 1; break; }
+            while (ld_acquire(p.flags + (int64_t)(flag_base + e) * p.flag_stride) != p.epoch) {
+                if (++it > kWaitLimit) { fail = true; break; }
                 __nanosleep(64);
             }
-            if (s_abort) break;
+        }
+        if (__any_sync(0xffffffffu, fail) && tid == 0) {
+            atomicOr(p.err, kErrWait);
+            s_abort = 1;
         }
     }
     __syncthreads();
@@ -294,6 +304,7 @@ extern "C" kvm_status kvm_kv_compact_noalloc(void* K, void* V, int32_t* position
     p.pos = positions;
     p.tickets = reinterpret_cast<int32_t*>(tickets);
     p.flags = flags;
+    p.flag_stride = 1;
     p.err = reinterpret_cast<int32_t*>(scratch);
     CompactChar& c = p.ch[0];
     c.L_new = L_new;

@@ -54,7 +54,8 @@ kvm_status fail(kvm_status code, const char* fmt, ...) {
 int attention_grid_cap(int num_sms, int head_dim) {
     return std::max(1, std::min(kMaxAttnCtas, num_sms * attention_ctas_per_sm(head_dim)));
 }
-constexpr int kMinUnitsPerCta = 4;  // smallest share of (query tile, key tile) units per attention block
+constexpr int kMinUnitsPerCta = 4;
+constexpr int kFlagStride = 32;     // compaction read flags: one per 128-byte line  // smallest share of (query tile, key tile) units per attention block
 
 }  // namespace
 
@@ -295,7 +296,7 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
     if (e == cudaSuccess) e = alloc_zero(&c->part_o, part_slots * kAttnRows * c->D);
     if (e == cudaSuccess) e = alloc_zero(&c->part_ml, part_slots * kAttnRows * 2);
     if (e == cudaSuccess) e = alloc_zero(&c->tickets, (size_t)n_chars * (n_kv_slabs + 1));
-    if (e == cudaSuccess) e = alloc_zero(&c->flags, n_flags);
+    if (e == cudaSuccess) e = alloc_zero(&c->flags, n_flags * kFlagStride);
     if (e == cudaSuccess) e = alloc_zero(&c->err, 1);
     if (e == cudaSuccess) e = alloc_zero(&c->diag, 16);
     if (c->n_gdn > 0) {
@@ -506,6 +507,7 @@ kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, c
         p.pos = c->pos;
         p.tickets = c->tickets;
         p.flags = c->flags;
+        p.flag_stride = kFlagStride;
         p.err = c->err;
         int blk = 0;
         for (int b = 0; b < c->B; ++b) {

@@ -74,7 +74,8 @@ struct CompactParams {
     uint4* V;
     int32_t* pos;
     int32_t* tickets;     // [n_chars][n_kv_slabs + 1]
-    uint32_t* flags;
+    uint32_t* flags;      // read flag of chunk i at flags[i * flag_stride]
+    int32_t flag_stride;  // 32 keeps every flag in its own 128-byte line (no line shared by pollers)
     int32_t* err;
     CompactChar ch[kMaxChars];
     // segment k of a character: survivors whose new index is >= seg_start[k]
