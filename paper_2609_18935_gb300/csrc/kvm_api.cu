@@ -54,8 +54,8 @@ kvm_status fail(kvm_status code, const char* fmt, ...) {
 int attention_grid_cap(int num_sms, int head_dim) {
     return std::max(1, std::min(kMaxAttnCtas, num_sms * attention_ctas_per_sm(head_dim)));
 }
-constexpr int kMinUnitsPerCta = 4;
-constexpr int kFlagStride = 32;     // compaction read flags: one per 128-byte line  // smallest share of (query tile, key tile) units per attention block
+constexpr int kMinUnitsPerCta = 4;  // smallest share of (query tile, key tile) units per attention block
+constexpr int kFlagStride = 32;     // compaction read flags: one per 128-byte line
 
 }  // namespace
 
@@ -94,11 +94,15 @@ struct kvm_ctx {
     int32_t* diag = nullptr;              // [16]: where the first expired device wait gave up
     uint8_t* gdn_work = nullptr;          // delta-rule prep records
     int64_t gdn_rec = 0;
-    // staging for host-resident round inputs
-    void* stage_in[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
-    void* stage_out = nullptr;
-    size_t stage_bytes[5] = {0, 0, 0, 0, 0};
-    size_t stage_out_bytes = 0;
+    // staging for host-resident rounds: every layer's inputs (q, k, v, alpha,
+    // beta) and output have their own buffers, so the copies of all layers
+    // run on a copy stream beside the kernels
+    uint8_t* stage = nullptr;
+    std::vector<size_t> stage_in_off;     // [n_layers * 5]
+    std::vector<size_t> stage_out_off;    // [n_layers]
+    cudaStream_t copy_stream = nullptr;
+    cudaEvent_t ev_start = nullptr, ev_copies = nullptr;
+    std::vector<cudaEvent_t> ev_in, ev_done;   // per layer: inputs landed, outputs written
     double inv_freq[kMaxRotaryHalf] = {};
     CUtensorMap tmap_q, tmap_k, tmap_v;   // TMA maps of q_rot, K, V (attention layers only)
     int64_t launches = 0;
@@ -122,10 +126,14 @@ cudaError_t alloc_zero(T** p, size_t count) {
 
 void free_all(kvm_ctx* c) {
     void* ptrs[] = {c->K, c->V, c->pos, c->S, c->q_rot, c->part_o, c->part_ml, c->tickets,
-                    c->flags, c->err, c->stage_in[0], c->stage_in[1], c->stage_in[2],
-                    c->stage_in[3], c->stage_in[4], c->stage_out, c->gdn_work, c->diag};
+                    c->flags, c->err, c->stage, c->gdn_work, c->diag};
     for (void* p : ptrs)
         if (p) cudaFree(p);
+    for (cudaEvent_t e : c->ev_in) if (e) cudaEventDestroy(e);
+    for (cudaEvent_t e : c->ev_done) if (e) cudaEventDestroy(e);
+    if (c->ev_start) cudaEventDestroy(c->ev_start);
+    if (c->ev_copies) cudaEventDestroy(c->ev_copies);
+    if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
     for (cudaEvent_t e : c->ev) cudaEventDestroy(e);
     c->ev.clear();
 }
@@ -282,10 +290,6 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         n_flags += (size_t)n_kv_slabs * ((c->cap[b] + c->rows_kv - 1) / c->rows_kv) +
                    (c->cap[b] + c->rows_pos - 1) / c->rows_pos;
     }
-    const size_t attn_in = (size_t)max_tail_tokens * std::max(c->Hq * c->D, c->H * c->dk);
-    const size_t kv_in = (size_t)max_tail_tokens * std::max(c->Hkv * c->D, c->H * c->dk);
-    const size_t v_in = (size_t)max_tail_tokens * std::max(c->Hkv * c->D, c->H * c->dv);
-    const size_t out_n = (size_t)max_tail_tokens * std::max(c->Hq * c->D, c->H * c->dv);
     e = cudaSuccess;
     if (e == cudaSuccess) e = alloc_zero(&c->K, kv_elems);
     if (e == cudaSuccess) e = alloc_zero(&c->V, kv_elems);
@@ -305,15 +309,30 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         const size_t chunks = (size_t)max_tail_tokens / 64 + n_chars;
         if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&c->gdn_work), chunks * c->H * c->gdn_rec);
     }
-    c->stage_bytes[0] = attn_in * 2;   // q
-    c->stage_bytes[1] = kv_in * 2;     // k
-    c->stage_bytes[2] = v_in * 2;      // v
-    c->stage_bytes[3] = (size_t)max_tail_tokens * std::max(c->H, 1) * 4;   // alpha
-    c->stage_bytes[4] = c->stage_bytes[3];                                  // beta
-    c->stage_out_bytes = out_n * 2;
-    for (int i = 0; i < 5 && e == cudaSuccess; ++i)
-        e = cudaMalloc(&c->stage_in[i], c->stage_bytes[i]);
-    if (e == cudaSuccess) e = cudaMalloc(&c->stage_out, c->stage_out_bytes);
+    {
+        size_t total_stage = 0;
+        auto take = [&](size_t bytes) { const size_t off = total_stage; total_stage += (bytes + 255) / 256 * 256; return off; };
+        const size_t T = (size_t)max_tail_tokens;
+        for (int l = 0; l < c->n_layers; ++l) {
+            const bool attn = c->kind[l] == KVM_LAYER_ATTN;
+            c->stage_in_off.push_back(take(T * (attn ? c->Hq * c->D : c->H * c->dk) * 2));    // q
+            c->stage_in_off.push_back(take(T * (attn ? c->Hkv * c->D : c->H * c->dk) * 2));   // k
+            c->stage_in_off.push_back(take(T * (attn ? c->Hkv * c->D : c->H * c->dv) * 2));   // v
+            c->stage_in_off.push_back(attn ? 0 : take(T * c->H * 4));                        // alpha
+            c->stage_in_off.push_back(attn ? 0 : take(T * c->H * 4));                        // beta
+            c->stage_out_off.push_back(take(T * (attn ? c->Hq * c->D : c->H * c->dv) * 2));  // out
+        }
+        if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&c->stage), total_stage);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_start, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_copies, cudaEventDisableTiming);
+        c->ev_in.assign(c->n_layers, nullptr);
+        c->ev_done.assign(c->n_layers, nullptr);
+        for (int l = 0; l < c->n_layers && e == cudaSuccess; ++l) {
+            e = cudaEventCreateWithFlags(&c->ev_in[l], cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_done[l], cudaEventDisableTiming);
+        }
+    }
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         free_all(c);
@@ -807,36 +826,65 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
                 return fail(KVM_E_INVAL, "layer %d has NULL gates", l);
         }
     }
+    const bool host_io = r->io_on_host && total > 0;
+    auto sizes = [&](int l, size_t n[6]) {
+        const bool attn = c->kind[l] == KVM_LAYER_ATTN;
+        n[0] = (size_t)total * (attn ? c->Hq * c->D : c->H * c->dk) * 2;
+        n[1] = (size_t)total * (attn ? c->Hkv * c->D : c->H * c->dk) * 2;
+        n[2] = (size_t)total * (attn ? c->Hkv * c->D : c->H * c->dv) * 2;
+        n[3] = n[4] = attn ? 0 : (size_t)total * c->H * 4;
+        n[5] = (size_t)total * (attn ? c->Hq * c->D : c->H * c->dv) * 2;
+    };
+    if (host_io) {
+        // every layer's inputs go up on the copy stream at once (after the work
+        // already queued on s, which may still read the staging buffers)
+        CUDA_TRY(cudaEventRecord(c->ev_start, s));
+        CUDA_TRY(cudaStreamWaitEvent(c->copy_stream, c->ev_start, 0));
+        for (int l = 0; l < c->n_layers; ++l) {
+            size_t n[6];
+            sizes(l, n);
+            const void* src[5] = {r->q[l], r->k[l], r->v[l], r->alpha ? r->alpha[l] : nullptr,
+                                  r->beta ? r->beta[l] : nullptr};
+            for (int i = 0; i < 5; ++i)
+                if (n[i]) CUDA_TRY(cudaMemcpyAsync(c->stage + c->stage_in_off[5 * l + i], src[i], n[i],
+                                                   cudaMemcpyHostToDevice, c->copy_stream));
+            CUDA_TRY(cudaEventRecord(c->ev_in[l], c->copy_stream));
+        }
+    }
     st = do_compact(c, r->span_cu, r->span_begin, r->span_end, r->gather_out, s);
     if (st) return st;
     for (int l = 0; l < c->n_layers; ++l) {
         const bool attn = c->kind[l] == KVM_LAYER_ATTN;
-        const size_t nq = (size_t)total * (attn ? c->Hq * c->D : c->H * c->dk) * 2;
-        const size_t nk = (size_t)total * (attn ? c->Hkv * c->D : c->H * c->dk) * 2;
-        const size_t nv = (size_t)total * (attn ? c->Hkv * c->D : c->H * c->dv) * 2;
-        const size_t ng = (size_t)total * c->H * 4;
-        const size_t no = (size_t)total * (attn ? c->Hq * c->D : c->H * c->dv) * 2;
         const void *q = r->q[l], *k = r->k[l], *v = r->v[l];
         const float *al = attn ? nullptr : r->alpha[l], *be = attn ? nullptr : r->beta[l];
         void* out = r->out[l];
-        if (r->io_on_host && total > 0) {
-            CUDA_TRY(cudaMemcpyAsync(c->stage_in[0], q, nq, cudaMemcpyHostToDevice, s));
-            CUDA_TRY(cudaMemcpyAsync(c->stage_in[1], k, nk, cudaMemcpyHostToDevice, s));
-            CUDA_TRY(cudaMemcpyAsync(c->stage_in[2], v, nv, cudaMemcpyHostToDevice, s));
-            q = c->stage_in[0]; k = c->stage_in[1]; v = c->stage_in[2];
+        if (host_io) {
+            CUDA_TRY(cudaStreamWaitEvent(s, c->ev_in[l], 0));
+            const size_t* o = &c->stage_in_off[5 * l];
+            q = c->stage + o[0]; k = c->stage + o[1]; v = c->stage + o[2];
             if (!attn) {
-                CUDA_TRY(cudaMemcpyAsync(c->stage_in[3], al, ng, cudaMemcpyHostToDevice, s));
-                CUDA_TRY(cudaMemcpyAsync(c->stage_in[4], be, ng, cudaMemcpyHostToDevice, s));
-                al = static_cast<const float*>(c->stage_in[3]);
-                be = static_cast<const float*>(c->stage_in[4]);
+                al = reinterpret_cast<const float*>(c->stage + o[3]);
+                be = reinterpret_cast<const float*>(c->stage + o[4]);
             }
-            out = c->stage_out;
+            out = c->stage + c->stage_out_off[l];
         }
         st = attn ? do_attention(c, l, r->tail_cu, q, k, v, out, s)
                   : do_gdn(c, l, r->tail_cu, q, k, v, al, be, out, s);
         if (st) return st;
-        if (r->io_on_host && total > 0)
-            CUDA_TRY(cudaMemcpyAsync(r->out[l], c->stage_out, no, cudaMemcpyDeviceToHost, s));
+        if (host_io) {
+            // the layer's output goes down while the next layers compute
+            size_t n[6];
+            sizes(l, n);
+            CUDA_TRY(cudaEventRecord(c->ev_done[l], s));
+            CUDA_TRY(cudaStreamWaitEvent(c->copy_stream, c->ev_done[l], 0));
+            CUDA_TRY(cudaMemcpyAsync(r->out[l], c->stage + c->stage_out_off[l], n[5], cudaMemcpyDeviceToHost,
+                                     c->copy_stream));
+        }
+    }
+    if (host_io) {
+        // work queued on s after this round also follows the copies
+        CUDA_TRY(cudaEventRecord(c->ev_copies, c->copy_stream));
+        CUDA_TRY(cudaStreamWaitEvent(s, c->ev_copies, 0));
     }
     do_advance(c, r->tail_cu);
     return KVM_OK;

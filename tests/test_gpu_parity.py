@@ -180,3 +180,55 @@ def test_spans_from_positions():
     assert list(sb) == [5, 40] and list(se) == [10, 41]
     with pytest.raises(kvm.KvmError):
         pair.ctx.spans_from_positions(0, [0], [10])     # covers no live entry
+
+
+def test_host_resident_round_equals_device_round():
+    """kvm_update_round with host-resident (pinned) inputs and outputs runs
+    the same kernels as with device tensors: outputs, caches and states
+    bit-identical, over two chained rounds of a 2-character population."""
+    import torch
+    from paper_2609_18935_gb300 import kvm
+    shape = W.ModelShape([W.GDN, W.ATTN, W.GDN, W.ATTN], 8, 2, 128, 64, 1e4, 4, 64, 96)
+    prefix = [300, 517]
+    caps = [640, 768]
+    w = W.Workload("host-io", 61, shape, prefix, 2)
+    w.plan = [[(0.05, 2, 70), (0.03, 1, 133)], [(0.02, 1, 64), (0.04, 3, 1)]]
+    mk = lambda: kvm.Context(shape.layer_kind, shape.n_q_heads, shape.n_kv_heads, shape.head_dim,
+                             shape.rotary_dim, shape.rope_theta, shape.n_gdn_heads, shape.d_k, shape.d_v, caps, 256)
+    N = sum(prefix)
+    ins = W.device_round_inputs(w, 7, prefix)
+    outs = {l: torch.empty((N, shape.n_q_heads, shape.head_dim) if k == W.ATTN else (N, shape.n_gdn_heads, shape.d_v),
+                           dtype=torch.bfloat16, device="cuda") for l, k in enumerate(shape.layer_kind)}
+    root2 = kvm.Context(shape.layer_kind, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.rotary_dim,
+                        shape.rope_theta, shape.n_gdn_heads, shape.d_k, shape.d_v, caps, N)
+    root2.update_round(np.zeros(3, np.int32), [], [], np.array([0, prefix[0], N], np.int32), ins, outs)
+    root2.check()
+    dev, host = mk(), mk()
+    dev.fork_from(root2)
+    host.fork_from(root2)
+    live = list(prefix)
+    for r in range(2):
+        span_cu, sb, se, tails = W.round_plan(w, r, live)
+        tail_cu = np.concatenate([[0], np.cumsum(tails)]).astype(np.int32)
+        T = int(tail_cu[-1])
+        d_in = W.device_round_inputs(w, 100 + r, tails)
+        h_in = {l: {k: t.cpu().pin_memory() for k, t in x.items()} for l, x in d_in.items()}
+        shp = lambda l: (T, shape.n_q_heads, shape.head_dim) if shape.layer_kind[l] == W.ATTN else (T, shape.n_gdn_heads, shape.d_v)
+        d_out = {l: torch.empty(shp(l), dtype=torch.bfloat16, device="cuda") for l in range(len(shape.layer_kind))}
+        h_out = {l: torch.empty(shp(l), dtype=torch.bfloat16).pin_memory() for l in range(len(shape.layer_kind))}
+        dev.update_round(span_cu, sb, se, tail_cu, d_in, d_out)
+        host.update_round(span_cu, sb, se, tail_cu, h_in, h_out, io_on_host=True)
+        dev.check()
+        host.check()
+        for l in range(len(shape.layer_kind)):
+            assert torch.equal(d_out[l].cpu().view(torch.int16), h_out[l].view(torch.int16)), (r, l)
+            if shape.layer_kind[l] == W.GDN:
+                assert torch.equal(dev.get_state(l).cpu(), host.get_state(l).cpu()), (r, l)
+            else:
+                for b in range(2):
+                    kd, vd = dev.get_kv(l, b)
+                    kh, vh = host.get_kv(l, b)
+                    assert torch.equal(kd.view(torch.int16), kh.view(torch.int16)) and torch.equal(
+                        vd.view(torch.int16), vh.view(torch.int16)), (r, l, b)
+        live = [dev.get_live(b)[0] for b in range(2)]
+        assert live == [host.get_live(b)[0] for b in range(2)]
