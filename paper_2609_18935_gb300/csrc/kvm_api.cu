@@ -55,6 +55,7 @@ int attention_grid_cap(int num_sms, int head_dim) {
     return std::max(1, std::min(kMaxAttnCtas, num_sms * attention_ctas_per_sm(head_dim)));
 }
 constexpr int kMinUnitsPerCta = 4;  // smallest share of (query tile, key tile) units per attention block
+constexpr double kSegmentCost = 8.0; // extra cost, in 64-key units, of each segment an attention block starts
 constexpr int kFlagStride = 32;     // compaction read flags: one per 128-byte line
 
 }  // namespace
@@ -655,29 +656,61 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
             units += (int64_t)c->Hkv * ((ch.L_prev + std::min(ch.M, (qt + 1) * tpt) + 63) / 64);
     }
     p.n_tiles = tiles;
-    // stream-K: block cc processes units [cc U / G, (cc + 1) U / G), located
-    // as (query tile, key tile) by one walk over the tiles
+    // stream-K with a cost model: block cc gets a contiguous range of
+    // (query tile, key tile) units; a unit costs 1 and every segment a block
+    // starts (its first one, and each query tile it enters) costs
+    // kSegmentCost more (Q staging, the epilogue, the pipeline refill).  The
+    // ranges are cut greedily at a per-block cost target, found by bisection
+    // so that exactly G blocks cover the units with the least maximum cost.
     const int G = (int)std::max<int64_t>(1, std::min<int64_t>(attention_grid_cap(c->num_sms, c->D),
                                                               units / kMinUnitsPerCta));
     p.n_ctas = G;
     {
-        int cc = 0, t = 0;
-        int64_t base = 0;
-        for (int b = 0; b < c->B && cc < G; ++b) {
+        std::vector<int> nk_of;
+        nk_of.reserve(tiles);
+        for (int b = 0; b < c->B; ++b) {
             const AttnChar& ch = p.ch[b];
-            for (int h = 0; h < c->Hkv && cc < G; ++h)
-                for (int qt = 0; qt < ch.n_qtiles && cc < G; ++qt, ++t) {
-                    const int nk = (ch.L_prev + std::min(ch.M, (qt + 1) * tpt) + 63) / 64;
-                    while (cc < G && (int64_t)cc * units / G < base + nk) {
-                        p.cta_tile[cc] = t;
-                        p.cta_k[cc] = (int)((int64_t)cc * units / G - base);
-                        ++cc;
-                    }
-                    base += nk;
-                }
+            for (int h = 0; h < c->Hkv; ++h)
+                for (int qt = 0; qt < ch.n_qtiles; ++qt)
+                    nk_of.push_back((ch.L_prev + std::min(ch.M, (qt + 1) * tpt) + 63) / 64);
         }
-        p.cta_tile[G] = tiles;
-        p.cta_k[G] = 0;
+        // blocks needed to cover everything with ranges of cost <= target; the
+        // cut points go to p.cta_tile / p.cta_k when `emit`
+        auto cover = [&](double target, bool emit) -> int {
+            int blocks = 1;
+            double cost = kSegmentCost;
+            if (emit) { p.cta_tile[0] = 0; p.cta_k[0] = 0; }
+            for (int t = 0; t < (int)nk_of.size(); ++t) {
+                int k = 0;
+                if (t > 0) cost += kSegmentCost;                  // entering a new query tile
+                while (k < nk_of[t]) {
+                    const double room = target - cost;
+                    const int take = room >= nk_of[t] - k ? nk_of[t] - k : std::max(0, (int)room);
+                    k += take;
+                    cost += take;
+                    if (k < nk_of[t] && (take == 0 || cost >= target)) {
+                        if (take == 0 && cost == kSegmentCost) {      // a block must take at least a unit
+                            ++k;
+                            cost += 1;
+                            if (k >= nk_of[t]) break;
+                        }
+                        if (emit && blocks <= G) { p.cta_tile[blocks] = t; p.cta_k[blocks] = k; }
+                        ++blocks;
+                        cost = kSegmentCost;
+                    }
+                }
+            }
+            return blocks;
+        };
+        double lo = (double)units / G, hi = (double)units / G + 2.0 * kSegmentCost * (1 + tiles / G) + 1.0;
+        while (cover(hi, false) > G) hi *= 2;
+        for (int it = 0; it < 40 && hi - lo > 0.25; ++it) {
+            const double mid = 0.5 * (lo + hi);
+            if (cover(mid, false) <= G) hi = mid; else lo = mid;
+        }
+        const int used = cover(hi, true);
+        // fewer ranges than blocks: the spare blocks get empty ranges at the end
+        for (int cc = used; cc <= G; ++cc) { p.cta_tile[cc] = tiles; p.cta_k[cc] = 0; }
     }
     // tiles shared by several blocks: each is merged once, from the first
     // block that starts inside it
