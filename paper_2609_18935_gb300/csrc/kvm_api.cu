@@ -103,6 +103,10 @@ struct kvm_ctx {
     std::vector<size_t> stage_out_off;    // [n_layers]
     cudaStream_t copy_stream = nullptr;
     cudaEvent_t ev_start = nullptr, ev_copies = nullptr;
+    // a round's compaction runs on its own stream beside the recurrent layers
+    // that come before the first attention layer (it touches only the KV cache)
+    cudaStream_t compact_stream = nullptr;
+    cudaEvent_t ev_round = nullptr, ev_compacted = nullptr;
     std::vector<cudaEvent_t> ev_in, ev_done;   // per layer: inputs landed, outputs written
     double inv_freq[kMaxRotaryHalf] = {};
     CUtensorMap tmap_q, tmap_k, tmap_v;   // TMA maps of q_rot, K, V (attention layers only)
@@ -135,6 +139,9 @@ void free_all(kvm_ctx* c) {
     if (c->ev_start) cudaEventDestroy(c->ev_start);
     if (c->ev_copies) cudaEventDestroy(c->ev_copies);
     if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
+    if (c->ev_round) cudaEventDestroy(c->ev_round);
+    if (c->ev_compacted) cudaEventDestroy(c->ev_compacted);
+    if (c->compact_stream) cudaStreamDestroy(c->compact_stream);
     for (cudaEvent_t e : c->ev) cudaEventDestroy(e);
     c->ev.clear();
 }
@@ -327,6 +334,9 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_start, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_copies, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->compact_stream, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_round, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_compacted, cudaEventDisableTiming);
         c->ev_in.assign(c->n_layers, nullptr);
         c->ev_done.assign(c->n_layers, nullptr);
         for (int l = 0; l < c->n_layers && e == cudaSuccess; ++l) {
@@ -884,10 +894,35 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
             CUDA_TRY(cudaEventRecord(c->ev_in[l], c->copy_stream));
         }
     }
-    st = do_compact(c, r->span_cu, r->span_begin, r->span_end, r->gather_out, s);
-    if (st) return st;
+    // Compaction changes only the attention layers' caches.  With recurrent
+    // layers ahead of the first attention layer it runs on the compaction
+    // stream beside them (after everything already queued on s), and s joins
+    // it one layer early, so the join never stalls the stream and breaks the
+    // launch overlap of a kernel that waits anyway.
+    int first_attn = c->n_layers;
+    for (int l = c->n_layers - 1; l >= 0; --l)
+        if (c->kind[l] == KVM_LAYER_ATTN) first_attn = l;
+    const bool side = first_attn > 0 && first_attn < c->n_layers;
+    const int join_at = first_attn >= 2 ? first_attn - 1 : first_attn;
+    if (side) {
+        CUDA_TRY(cudaEventRecord(c->ev_round, s));
+        CUDA_TRY(cudaStreamWaitEvent(c->compact_stream, c->ev_round, 0));
+        st = do_compact(c, r->span_cu, r->span_begin, r->span_end, r->gather_out, c->compact_stream);
+        if (st) return st;
+        CUDA_TRY(cudaEventRecord(c->ev_compacted, c->compact_stream));
+    } else {
+        st = do_compact(c, r->span_cu, r->span_begin, r->span_end, r->gather_out, s);
+        if (st) return st;
+    }
+    bool joined = !side;
+    auto join = [&]() -> cudaError_t {
+        if (joined) return cudaSuccess;
+        joined = true;
+        return cudaStreamWaitEvent(s, c->ev_compacted, 0);
+    };
     for (int l = 0; l < c->n_layers; ++l) {
         const bool attn = c->kind[l] == KVM_LAYER_ATTN;
+        if (l == join_at) CUDA_TRY(join());
         const void *q = r->q[l], *k = r->k[l], *v = r->v[l];
         const float *al = attn ? nullptr : r->alpha[l], *be = attn ? nullptr : r->beta[l];
         void* out = r->out[l];
@@ -903,7 +938,10 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
         }
         st = attn ? do_attention(c, l, r->tail_cu, q, k, v, out, s)
                   : do_gdn(c, l, r->tail_cu, q, k, v, al, be, out, s);
-        if (st) return st;
+        if (st) {
+            join();                                   // s still covers the compaction
+            return st;
+        }
         if (host_io) {
             // the layer's output goes down while the next layers compute
             size_t n[6];

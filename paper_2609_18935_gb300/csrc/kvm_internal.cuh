@@ -139,7 +139,7 @@ struct AttnParams {
     __nv_bfloat16* V;
     int32_t* pos;                 // [slab_rows]
     __nv_bfloat16* out;           // [sum M][Hq][D]
-    float* part_o;                // [2 n_ctas][D / 32][128][32]: partial O of a block's first / last segment
+    float* part_o;                // [2 n_ctas][D / 32][8][128][4]: partial O of a block's first / last segment
     float* part_ml;               // [2 n_ctas][128][2]: (reference max in log2 units, sum) of a partial
     int32_t* err;
     int32_t* diag;                // first expired wait: block + 1, tag, parity

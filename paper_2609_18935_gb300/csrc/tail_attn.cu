@@ -167,9 +167,10 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
 // inside the tile, so its partials are in the slots of blocks c0 = cb - 1 ..
 // c1 (the last block that starts inside the tile): c0's last segment (slot
 // 2 c0 + 1, or 2 c0 when the tile is also c0's first segment) and the first
-// segments 2 c of the others.  A thread owns four columns of one row and
-// merges the partials online, eight at a time, each batch's (max, sum) pairs
-// and O pieces loaded together.
+// segments 2 c of the others.  A thread owns four columns of one row (rows
+// fastest across threads, as in the partial layout) and merges the partials
+// online, eight at a time, each batch's (max, sum) pairs and O pieces loaded
+// together.
 __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant__ AttnParams p) {
     grid_dependency_wait();
     grid_dependents_launch();
@@ -192,10 +193,10 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
     const int kvh = local / c.n_qtiles, qt = local % c.n_qtiles;
     const int D = p.D;
     const int groups = D / 32;                                     // 32-column groups
-    const int item = blockIdx.y * blockDim.x + threadIdx.x;        // (row, 4-column piece)
-    const int r = item / (D / 4);
-    if (r >= kRows) return;
-    const int piece = item % (D / 4);
+    const int item = blockIdx.y * blockDim.x + threadIdx.x;        // (4-column piece, row): rows fastest
+    const int r = item % kRows;
+    const int piece = item / kRows;
+    if (piece >= D / 4) return;
     const int cg = piece >> 3, q4 = piece & 7;
     const int tok = qt * p.tok_per_tile + r / p.g;
     if (tok >= c.M) return;
@@ -210,7 +211,7 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
             if (q0 + u < n_parts) {
                 const int64_t slot = slot_of(q0 + u);
                 ml[u] = *reinterpret_cast<const float2*>(p.part_ml + (slot * kRows + r) * 2);
-                x[u] = *reinterpret_cast<const float4*>(p.part_o + ((slot * groups + cg) * kRows + r) * 32 + q4 * 4);
+                x[u] = *reinterpret_cast<const float4*>(p.part_o + (((slot * groups + cg) * 8 + q4) * kRows + r) * 4);
             } else {
                 ml[u] = make_float2(-INFINITY, 0.f);
             }

@@ -468,7 +468,8 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
                     p.part_ml[prow * 2 + 0] = mr;
                     p.part_ml[prow * 2 + 1] = lt;
                 }
-                // partial layout [slot][D / 32][row][32]: a warp stores 4 KB contiguously
+                // partial layout [slot][D / 32][8][row][4]: each 16-byte store
+                // of a warp lands in 512 contiguous bytes
                 const int64_t slot = 2 * cta + (seg == 0 ? 0 : 1);
 #pragma unroll 1
                 for (int c0 = half * C::HALF; c0 < (half + 1) * C::HALF; c0 += 32) {
@@ -476,9 +477,10 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
                     tmem_ld32(tmem + lane_off + C::TMEM_O + c0, v);
                     tmem_ld_wait();
                     if (store) {
-                        uint4* dst = reinterpret_cast<uint4*>(p.part_o + ((slot * (D / 32) + c0 / 32) * BM + r) * 32);
+                        uint4* dst = reinterpret_cast<uint4*>(p.part_o + (slot * (D / 32) + c0 / 32) * 8 * BM * 4) + r;
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) dst[e] = make_uint4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+                        for (int e = 0; e < 8; ++e)
+                            dst[e * BM] = make_uint4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
                     }
                 }
             }
