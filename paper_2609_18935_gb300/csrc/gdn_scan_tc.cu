@@ -133,7 +133,13 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     const int row = q4 * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     const int H = p.H, dv = p.dv;
-    const int chunk = blockIdx.x / H, h = blockIdx.x % H;
+    // with two parts per (chunk, head) both solve for X; part 0 writes the
+    // [W; Q'] and K images, part 1 U | A U and w, G_C
+    const int part = blockIdx.x % p.prep_parts;
+    const int ch_h = blockIdx.x / p.prep_parts;
+    const bool do_w = p.prep_parts == 1 || part == 0;
+    const bool do_u = p.prep_parts == 1 || part == 1;
+    const int chunk = ch_h / H, h = ch_h % H;
     const int b = find_char_by_chunk(p, chunk);
     const GdnChar ch = p.ch[b];
     const int c0 = (chunk - ch.chunk_off) * C;
@@ -169,7 +175,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
         for (int u = 0; u < NV; ++u) {
             const int i = tid + u * kThreads;
             const int t = i / (dv / 8), r8 = (i % (dv / 8)) * 8;
-            vv[u] = (i < C * (dv / 8) && t < n) ? __ldg(reinterpret_cast<const uint4*>(p.v + ((tok0 + t) * H + h) * dv + r8))
+            vv[u] = (do_u && i < C * (dv / 8) && t < n) ? __ldg(reinterpret_cast<const uint4*>(p.v + ((tok0 + t) * H + h) * dv + r8))
                                                 : make_uint4(0, 0, 0, 0);
         }
 #pragma unroll
@@ -181,7 +187,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
 #pragma unroll
         for (int u = 0; u < NV; ++u) {
             const int i = tid + u * kThreads;
-            if (i < C * (dv / 8)) V4(oV + sw128_off16(i / (dv / 8), (i % (dv / 8)) * 8, C)) = vv[u];
+            if (do_u && i < C * (dv / 8)) V4(oV + sw128_off16(i / (dv / 8), (i % (dv / 8)) * 8, C)) = vv[u];
         }
     }
     if (tid < 32) {
@@ -207,9 +213,11 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     if (tid < C) {
         Gs[tid] = expf(gs[tid]);
         g2[tid] = gs[tid] * 1.4426950408889634f;          // log2 domain for the decays
-        float* misc = reinterpret_cast<float*>(rec + R::misc_off(dv));
-        misc[tid] = tid < n ? bs[tid] * expf(gs[n - 1] - gs[tid]) : 0.f;     // w_j
-        if (tid == 0) misc[C] = expf(gs[n - 1]);                            // G_C
+        if (do_u) {
+            float* misc = reinterpret_cast<float*>(rec + R::misc_off(dv));
+            misc[tid] = tid < n ? bs[tid] * expf(gs[n - 1] - gs[tid]) : 0.f;     // w_j
+            if (tid == 0) misc[C] = expf(gs[n - 1]);                            // G_C
+        }
     }
     uint32_t phase = 0;
     bool ok = true;
@@ -399,12 +407,16 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
             }
             uint4 hi, lo;
             const uint32_t off = sw128_off16(row, hf * 32 + j8, 128);
-            split8(xg, hi, lo);
-            V4(oXG + off) = hi;
-            V4(oXG + T128 + off) = lo;
-            split8(xr, hi, lo);
-            V4(oX + off) = hi;
-            V4(oX + T128 + off) = lo;
+            if (do_w) {
+                split8(xg, hi, lo);
+                V4(oXG + off) = hi;
+                V4(oXG + T128 + off) = lo;
+            }
+            if (do_u) {
+                split8(xr, hi, lo);
+                V4(oX + off) = hi;
+                V4(oX + T128 + off) = lo;
+            }
         }
     }
     fence_proxy_async_smem();
@@ -418,12 +430,14 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
             const uint64_t bk = smem_desc_sw128(sb + oKQ + ks * 2048, kq_region, 1024);
             const uint64_t bvv = smem_desc_sw128(sb + oV + ks * 2048, C * 128, 1024);
 #pragma unroll
-            for (int part = 0; part < 2; ++part) {
-                const uint32_t ao = part * T128 + ks * 32;
-                mma_bf16(tmem + G::T_WU, smem_desc_sw128(sb + oXG + ao, 16, 1024), bk,
-                         idesc_bf16_f32(128, DK, true), (ks | part) != 0);
-                mma_bf16(tmem + G::T_WU + DK, smem_desc_sw128(sb + oX + ao, 16, 1024), bvv,
-                         idesc_bf16_f32(128, dv, true), (ks | part) != 0);
+            for (int hl = 0; hl < 2; ++hl) {             // the hi and lo halves of the X operand
+                const uint32_t ao = hl * T128 + ks * 32;
+                if (do_w)
+                    mma_bf16(tmem + G::T_WU, smem_desc_sw128(sb + oXG + ao, 16, 1024), bk,
+                             idesc_bf16_f32(128, DK, true), (ks | hl) != 0);
+                if (do_u)
+                    mma_bf16(tmem + G::T_WU + DK, smem_desc_sw128(sb + oX + ao, 16, 1024), bvv,
+                             idesc_bf16_f32(128, dv, true), (ks | hl) != 0);
             }
         }
         mma_commit(mbar);
@@ -436,7 +450,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
         const int t = row & 63;
         const float gt = Gs[t];
         const uint32_t oWQ = G::OFF_STAGE_WQ;
-        for (int cb = hf * (DK / 2); cb < (hf + 1) * (DK / 2); cb += 32) {
+        for (int cb = hf * (DK / 2); do_w && cb < (hf + 1) * (DK / 2); cb += 32) {
             uint32_t v[32];
             tmem_ld32(tmem + lane_off + G::T_WU + cb, v);
             tmem_ld_wait();
@@ -469,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
         const int dh = ((dv / 2) + 31) / 32 * 32;
         const int nc = dv / 4;                               // 16-byte chunks per row
         const uint32_t urow = G::OFF_STAGE_U + (uint32_t)row * dv * 4;
-        for (int rc = hf * dh; rc < min(dv, (hf + 1) * dh); rc += 32) {
+        for (int rc = hf * dh; do_u && rc < min(dv, (hf + 1) * dh); rc += 32) {
             uint32_t v[32];
             tmem_ld32(tmem + lane_off + G::T_WU + DK + rc, v);
             tmem_ld_wait();
@@ -482,11 +496,13 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     fence_proxy_async_smem();
     __syncthreads();
     if (ok && tid == 0) {
-        bulk_store(rec, sb + G::OFF_STAGE_WQ, 2 * (uint32_t)R::WQH);
-        // K image: rows 0..63 of each 64-column region of [K;Q]
-        for (int r = 0; r < DK / 64; ++r)
-            bulk_store(rec + 2 * R::WQH + r * (64 * 128), sb + oKQ + r * (128 * 128), 64 * 128);
-        bulk_store(rec + R::uau_off(), sb + G::OFF_STAGE_U, 128u * dv * 4u);
+        if (do_w) {
+            bulk_store(rec, sb + G::OFF_STAGE_WQ, 2 * (uint32_t)R::WQH);
+            // K image: rows 0..63 of each 64-column region of [K;Q]
+            for (int r = 0; r < DK / 64; ++r)
+                bulk_store(rec + 2 * R::WQH + r * (64 * 128), sb + oKQ + r * (128 * 128), 64 * 128);
+        }
+        if (do_u) bulk_store(rec + R::uau_off(), sb + G::OFF_STAGE_U, 128u * dv * 4u);
         bulk_commit();
         // the sources must be read before the block's shared memory is
         // released; the writes complete with the grid, before the scan
@@ -809,7 +825,7 @@ void configure_once(int smem) {
 template <int DK>
 void launch_prep_dk(const GdnParams& p, cudaStream_t s) {
     configure_once<gdn_prep_kernel<DK>>(PrepCfg<DK>::SMEM);
-    launch_pdl(gdn_prep_kernel<DK>, dim3(p.total_chunks * p.H), dim3(kThreads), PrepCfg<DK>::SMEM, s, p);
+    launch_pdl(gdn_prep_kernel<DK>, dim3(p.total_chunks * p.H * p.prep_parts), dim3(kThreads), PrepCfg<DK>::SMEM, s, p);
 }
 
 template <int DK>

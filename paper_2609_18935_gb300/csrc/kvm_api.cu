@@ -790,6 +790,10 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
         chunks += (p.ch[b].M + 63) / 64;
     }
     p.total_chunks = chunks;
+    // two prep blocks per (chunk, head) when both fit on the SMs at once: they
+    // share the solve for X and halve the products, staging and record
+    // stores that follow it
+    p.prep_parts = (int64_t)2 * chunks * c->H <= c->num_sms ? 2 : 1;
     int ps = prof_begin(c, KVM_K_GDN_PREP, s);
     launch_gdn_chunk_prep(p, s);
     prof_end(c, ps, s);

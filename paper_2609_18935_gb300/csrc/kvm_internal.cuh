@@ -169,6 +169,7 @@ struct GdnChar {
 struct GdnParams {
     int32_t n_chars, H, dk, dv;
     int32_t dv_slice;         // rows of S per block (a multiple of 16, <= 128, dividing dv)
+    int32_t prep_parts;       // prep blocks per (chunk, head): 1, or 2 (one writes [W; Q'] and K, one U | A U)
     const __nv_bfloat16* q;   // [sum M][H][dk]
     const __nv_bfloat16* k;
     const __nv_bfloat16* v;   // [sum M][H][dv]
