@@ -449,7 +449,7 @@ def run_kvm(args):
     # ---- CPU oracle sample (rank 0 only, single GPU runs only)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        secs, m = oracle_sample(w, 64)
+        secs, m = oracle_sample(w, 256)
         cpu = {"value": m / secs, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
                "sample": f"character 0, round 0: compaction + all {len(s.layer_kind)} layers for the first "
                          f"{m} of {plan[0][3][0]} tail tokens (prefix {w.prefix_len[0]}), fp64 numpy, "
