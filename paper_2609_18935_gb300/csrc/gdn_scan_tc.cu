@@ -43,10 +43,12 @@ constexpr int DSTRIDE = 20;      // fp32 row stride of the diagonal-block invers
 // Workspace record of one (chunk, head):
 //   [W;Q'] hi | [W;Q'] lo   (128 x DK bf16 each, K-major 128-byte-swizzled image)
 //   K                       (64 x DK bf16, 128-byte-swizzled image, rows = tokens)
-//   U | A U                 (fp32 [128][dv], rows 0..63 U, 64..127 A U; the
-//                            16-byte chunk c of row r is stored at chunk
-//                            (c + r) mod (dv/4), so row-parallel reads of a
-//                            copy in shared memory do not collide on banks)
+//   U | A U                 (fp32, rows 0..63 U, 64..127 A U, in slices of 32
+//                            columns [dv/32][128][32]: a scan block's d_v rows are
+//                            one contiguous piece; within a slice the 16-byte
+//                            chunk c of row r sits at chunk (c + r) mod 8, so
+//                            row-parallel reads of a copy in shared memory do not
+//                            collide on banks)
 //   w[64], G_C              (fp32)
 template <int DK>
 struct Rec {
@@ -57,6 +59,11 @@ struct Rec {
     static __host__ __device__ int64_t misc_off(int dv) { return IMG + (int64_t)128 * dv * 4; }
     static __host__ __device__ int64_t bytes(int dv) { return IMG + (int64_t)128 * dv * 4 + 512; }
 };
+
+// Float offset of (row, col) in a U | A U copy of 32-column slices.
+__device__ __forceinline__ int uau_idx(int row, int col) {
+    return ((col >> 5) * 128 + row) * 32 + 4 * ((((col & 31) >> 2) + row) & 7) + (col & 3);
+}
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
     __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
@@ -481,16 +488,14 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
             }
         }
         const int dh = ((dv / 2) + 31) / 32 * 32;
-        const int nc = dv / 4;                               // 16-byte chunks per row
-        const uint32_t urow = G::OFF_STAGE_U + (uint32_t)row * dv * 4;
+        float* us = reinterpret_cast<float*>(smem + G::OFF_STAGE_U);
         for (int rc = hf * dh; do_u && rc < min(dv, (hf + 1) * dh); rc += 32) {
             uint32_t v[32];
             tmem_ld32(tmem + lane_off + G::T_WU + DK + rc, v);
             tmem_ld_wait();
 #pragma unroll
             for (int j4 = 0; j4 < 32; j4 += 4)
-                if (rc + j4 < dv)
-                    V4(urow + 16u * (((rc + j4) / 4 + row) % nc)) = make_uint4(v[j4], v[j4 + 1], v[j4 + 2], v[j4 + 3]);
+                *reinterpret_cast<uint4*>(us + uau_idx(row, rc + j4)) = make_uint4(v[j4], v[j4 + 1], v[j4 + 2], v[j4 + 3]);
         }
     }
     fence_proxy_async_smem();
@@ -566,8 +571,8 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     if (ch.M <= 0) return;                           // uniform per block; touches no memory
     const int H = p.H, dv = p.dv;
     const int nch = (ch.M + C - 1) / C;
-    const int nc = dv / 4;                           // 16-byte chunks of a U | A U row
-    const uint32_t ubytes = 128u * dv * 4u;
+    const uint32_t ubytes = 128u * dvs * 4u;         // the block's slice of U | A U
+    const int64_t uslice = R::uau_off() + (int64_t)r0 * 128 * 4;
     float* Sg = p.S + ((int64_t)b * H + h) * dv * DK;
     const int dhalf = ((dvs / 2) + 31) / 32 * 32;
     const int dlo = hf * dhalf, dhi = min(dvs, dlo + dhalf);
@@ -628,7 +633,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         mbar_arrive_expect_tx(bar_k, G::KI);
         bulk_load(sb + G::OFF_K, rec_of(0) + G::WQ, G::KI, bar_k);
         mbar_arrive_expect_tx(bar_u, ubytes);
-        bulk_load(sb + G::OFF_U, rec_of(0) + R::uau_off(), ubytes, bar_u);
+        bulk_load(sb + G::OFF_U, rec_of(0) + uslice, ubytes, bar_u);
     }
 
     uint32_t phase = 0;
@@ -697,8 +702,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
                 float u[32];
 #pragma unroll
                 for (int j4 = 0; j4 < 32; j4 += 4) {
-                    const int cg = (r0 + rc + j4) / 4;   // chunk of the record row
-                    const float4 f = *reinterpret_cast<const float4*>(Us + (int64_t)row * dv + 4 * ((cg + row) % nc));
+                    const float4 f = *reinterpret_cast<const float4*>(Us + uau_idx(row, rc + j4));
                     u[j4] = f.x; u[j4 + 1] = f.y; u[j4 + 2] = f.z; u[j4 + 3] = f.w;
                 }
                 tmem_ld_wait();
@@ -740,7 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         issue_begin();
         if (tid == 0 && i + 1 < nch) {               // U | A U consumed: fetch the next one
             mbar_arrive_expect_tx(bar_u, ubytes);
-            bulk_load(sb + G::OFF_U, rec_of(i + 1) + R::uau_off(), ubytes, bar_u);
+            bulk_load(sb + G::OFF_U, rec_of(i + 1) + uslice, ubytes, bar_u);
         }
         // ---------------------------------------------------------------- S^T += K^T (w E)
         ok = __syncthreads_and(mbar_wait(bar_k, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x53 + 256 * i));
