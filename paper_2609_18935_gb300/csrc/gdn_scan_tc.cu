@@ -541,7 +541,9 @@ struct ScanCfg {
     static constexpr uint32_t T_S = 128;                     // S^T (dv cols)
 };
 
-template <int DK>
+// CW: columns of the slice a thread handles per TMEM access (16 when the
+// slice is 32 wide, so that all eight warps share the elementwise phases)
+template <int DK, int CW>
 __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_constant__ GdnParams p) {
     using G = ScanCfg<DK>;
     using R = Rec<DK>;
@@ -574,7 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     const uint32_t ubytes = 128u * dvs * 4u;         // the block's slice of U | A U
     const int64_t uslice = R::uau_off() + (int64_t)r0 * 128 * 4;
     float* Sg = p.S + ((int64_t)b * H + h) * dv * DK;
-    const int dhalf = ((dvs / 2) + 31) / 32 * 32;
+    const int dhalf = ((dvs / 2) + CW - 1) / CW * CW;
     const int dlo = hf * dhalf, dhi = min(dvs, dlo + dhalf);
     auto rec_of = [&](int i) -> const uint8_t* { return p.work + ((int64_t)(ch.chunk_off + i) * H + h) * p.rec_bytes; };
 
@@ -596,7 +598,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     const uint32_t tmem = *tmem_slot;
     auto write_s_row = [&](int c, int rc, const float* x) {
 #pragma unroll
-        for (int j8 = 0; j8 < 32; j8 += 8) {
+        for (int j8 = 0; j8 < CW; j8 += 8) {
             if (rc + j8 < dvs) {
                 uint4 hi, lo;
                 split8(x + j8, hi, lo);
@@ -609,16 +611,16 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     // ---- the state slice: S^T into TMEM (lane c, column r) and the MN-major operand
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
-        const int rc = dlo + 32 * half;
+        const int rc = dlo + CW * half;
         if (rc >= dhi) continue;                     // uniform per warp
-        float sx[32];
+        float sx[CW];
 #pragma unroll
-        for (int j = 0; j < 32; ++j)                 // all 32 loads before any use
+        for (int j = 0; j < CW; ++j)                 // all loads before any use
             sx[j] = (row < DK && rc + j < dhi) ? Sg[(int64_t)(r0 + rc + j) * DK + row] : 0.f;
-        uint32_t v[32];
+        uint32_t v[CW];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sx[j]);
-        tmem_st32(tmem + lane_off + G::T_S + rc, v);
+        for (int j = 0; j < CW; ++j) v[j] = __float_as_uint(sx[j]);
+        tmem_stw<CW>(tmem + lane_off + G::T_S + rc, v);
         if (row < DK) write_s_row(row, rc, sx);
     }
     tmem_st_wait();
@@ -694,24 +696,24 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
             const int t = row & 63;
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
-                const int rc = dlo + 32 * half;
+                const int rc = dlo + CW * half;
                 if (rc >= dhi) continue;                 // uniform per warp
-                uint32_t d1[32], sv[32];
-                tmem_ld32(tmem + lane_off + G::T_D + rc, d1);
-                tmem_ld32(tmem + lane_off + G::T_S + rc, sv);
-                float u[32];
+                uint32_t d1[CW], sv[CW];
+                tmem_ldw<CW>(tmem + lane_off + G::T_D + rc, d1);
+                tmem_ldw<CW>(tmem + lane_off + G::T_S + rc, sv);
+                float u[CW];
 #pragma unroll
-                for (int j4 = 0; j4 < 32; j4 += 4) {
+                for (int j4 = 0; j4 < CW; j4 += 4) {
                     const float4 f = *reinterpret_cast<const float4*>(Us + uau_idx(row, rc + j4));
                     u[j4] = f.x; u[j4 + 1] = f.y; u[j4 + 2] = f.z; u[j4 + 3] = f.w;
                 }
                 tmem_ld_wait();
                 if (row < 64) {
-                    float e[32];
+                    float e[CW];
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) e[j] = wt * (u[j] - __uint_as_float(d1[j]));
+                    for (int j = 0; j < CW; ++j) e[j] = wt * (u[j] - __uint_as_float(d1[j]));
 #pragma unroll
-                    for (int j8 = 0; j8 < 32; j8 += 8) {
+                    for (int j8 = 0; j8 < CW; j8 += 8) {
                         if (rc + j8 < dvs) {
                             uint4 hi, lo;
                             split8(e + j8, hi, lo);
@@ -723,7 +725,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
                 } else if (t < n) {
                     __nv_bfloat16* o = p.out + ((tok0 + t) * H + h) * dv + r0 + rc;
 #pragma unroll
-                    for (int j8 = 0; j8 < 32; j8 += 8) {
+                    for (int j8 = 0; j8 < CW; j8 += 8) {
                         if (rc + j8 < dvs) {
                             uint4 w4;
                             uint32_t* ww = reinterpret_cast<uint32_t*>(&w4);
@@ -736,8 +738,8 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
                     }
                 }
 #pragma unroll
-                for (int j = 0; j < 32; ++j) sv[j] = __float_as_uint(__uint_as_float(sv[j]) * gC);
-                tmem_st32(tmem + lane_off + G::T_S + rc, sv);
+                for (int j = 0; j < CW; ++j) sv[j] = __float_as_uint(__uint_as_float(sv[j]) * gC);
+                tmem_stw<CW>(tmem + lane_off + G::T_S + rc, sv);
             }
             tmem_st_wait();
         }
@@ -768,15 +770,15 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         // ---------------------------------------------------------------- refresh the state operand
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
-            const int rc = dlo + 32 * half;
+            const int rc = dlo + CW * half;
             if (rc >= dhi) continue;                     // uniform per warp
-            uint32_t sv[32];
-            tmem_ld32(tmem + lane_off + G::T_S + rc, sv);
+            uint32_t sv[CW];
+            tmem_ldw<CW>(tmem + lane_off + G::T_S + rc, sv);
             tmem_ld_wait();
             if (row < DK) {
-                float y[32];
+                float y[CW];
 #pragma unroll
-                for (int j = 0; j < 32; ++j) y[j] = __uint_as_float(sv[j]);
+                for (int j = 0; j < CW; ++j) y[j] = __uint_as_float(sv[j]);
                 write_s_row(row, rc, y);
             }
         }
@@ -785,14 +787,14 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     if (ok) {
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
-            const int rc = dlo + 32 * half;
+            const int rc = dlo + CW * half;
             if (rc >= dhi) continue;                     // uniform per warp
-            uint32_t sv[32];
-            tmem_ld32(tmem + lane_off + G::T_S + rc, sv);
+            uint32_t sv[CW];
+            tmem_ldw<CW>(tmem + lane_off + G::T_S + rc, sv);
             tmem_ld_wait();
             if (row < DK) {
 #pragma unroll
-                for (int j = 0; j < 32; ++j)
+                for (int j = 0; j < CW; ++j)
                     if (rc + j < dvs) Sg[(int64_t)(r0 + rc + j) * DK + row] = __uint_as_float(sv[j]);
             }
         }
@@ -832,11 +834,17 @@ void launch_prep_dk(const GdnParams& p, cudaStream_t s) {
     launch_pdl(gdn_prep_kernel<DK>, dim3(p.total_chunks * p.H * p.prep_parts), dim3(kThreads), PrepCfg<DK>::SMEM, s, p);
 }
 
+template <int DK, int CW>
+void launch_scan_cw(const GdnParams& p, cudaStream_t s) {
+    configure_once<gdn_scan_kernel<DK, CW>>(ScanCfg<DK>::SMEM);
+    dim3 grid(p.dv / p.dv_slice, p.H, p.n_chars);
+    launch_pdl(gdn_scan_kernel<DK, CW>, grid, dim3(kThreads), ScanCfg<DK>::SMEM, s, p);
+}
+
 template <int DK>
 void launch_scan_dk(const GdnParams& p, cudaStream_t s) {
-    configure_once<gdn_scan_kernel<DK>>(ScanCfg<DK>::SMEM);
-    dim3 grid(p.dv / p.dv_slice, p.H, p.n_chars);
-    launch_pdl(gdn_scan_kernel<DK>, grid, dim3(kThreads), ScanCfg<DK>::SMEM, s, p);
+    if (p.dv_slice <= 32) launch_scan_cw<DK, 16>(p, s);
+    else launch_scan_cw<DK, 32>(p, s);
 }
 
 }  // namespace
