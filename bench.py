@@ -60,6 +60,14 @@ def attention_flops(shape, Lp, tails):
     return sum(4.0 * D * Hq * (m * l + m * (m + 1) / 2) for l, m in zip(Lp, tails))
 
 
+def attention_bytes(shape, Lp, tails):
+    """K and V of the surviving keys once per KV head, q, k_new and v_new of
+    the tail, and the output, per attention layer."""
+    Hq, Hkv, D = shape.n_q_heads, shape.n_kv_heads, shape.head_dim
+    return float(sum(l for l, m in zip(Lp, tails) if m > 0) * Hkv * D * 2 * 2
+                 + sum(tails) * (2 * Hq + 2 * Hkv) * D * 2)
+
+
 def gdn_flops(shape, tails):
     return 6.0 * shape.d_k * shape.d_v * shape.n_gdn_heads * sum(tails)
 
@@ -332,6 +340,7 @@ def run_kvm(args):
                 moved += live[b] - rem - int(sb[cu[b]])
             live[b] = live[b] - rem + tails[b]
         rd["attn_flops"] = attention_flops(s, Lp, tails)        # per attention layer
+        rd["attn_bytes"] = attention_bytes(s, Lp, tails)        # per attention layer
         rd["gdn_flops"] = gdn_flops(s, tails)                   # per delta-rule layer
         rd["compact_bytes"] = compaction_bytes(s, moved)
         rd["gdn_bytes"] = gdn_bytes(s, tails)                   # per delta-rule layer
@@ -444,6 +453,21 @@ def run_kvm(args):
                                   else f"HBM copy bandwidth, {peak_src}"),
                     "traffic": ncu_traffic(kfile[dominant], dominant),
                     "algorithmic_per_launch": rf["per_launch"], "share_of_step": rf["share"]}
+    # round roofline: every kernel family at the larger of its tensor and HBM
+    # times (algorithmic work over the measured peaks), summed over the round
+    per_round = []
+    for r in rids:
+        rd = rounds[r]
+        t = n_attn * (max(rd["attn_flops"] / (tc_burst * 1e12), rd["attn_bytes"] / (hbm * 1e9))
+                      + rd["rope_bytes"] / (hbm * 1e9))
+        t += n_gdn * max(rd["gdn_flops"] / (tc_burst * 1e12), rd["gdn_bytes"] / (hbm * 1e9))
+        t += rd["compact_bytes"] / (hbm * 1e9)
+        per_round.append(t)
+    roof_us = 1e6 * sum(per_round) / len(per_round)
+    round_roofline = {"time_us": roof_us, "measured_us": 1e3 * total_ms / args.steps,
+                      "frac": roof_us / (1e3 * total_ms / args.steps),
+                      "model": "sum over the round's kernels of max(flops / bf16 peak, bytes / HBM peak), "
+                               f"algorithmic work, {peak_src} peaks"}
     if rank != 0:
         return
     # ---- CPU oracle sample (rank 0 only, single GPU runs only)
@@ -467,6 +491,7 @@ def run_kvm(args):
                    "l2": "flushed before every step (256 MiB write), outside the timed events",
                    "parallelism": f"{world} independent replica(s), characters per rank fixed"},
         "roofline": roofline,
+        "round_roofline": round_roofline,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT,
                 "h2d_bytes_per_step": int(np.mean([rounds[r]["h2d"] for r in e2e_rids])),
