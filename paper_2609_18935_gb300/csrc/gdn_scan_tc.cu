@@ -94,32 +94,36 @@ __device__ __forceinline__ int find_char_by_chunk(const GdnParams& p, int chunk)
 }
 
 // ============================================================================
-// prep: one block per (chunk, head)
+// prep: one block of 512 threads per (chunk, head) (or two, see prep_parts)
 // ============================================================================
+constexpr int kPrepThreads = 512;
+
 template <int DK>
 struct PrepCfg {
     static constexpr int KQ = 128 * DK * 2;                  // [K;Q] bf16, K-major, 128 rows
     static constexpr int V = C * DVP * 2;                    // V bf16, rows j (MN-major operand)
     static constexpr int TILE128 = 128 * 64 * 2;             // 128 x 64 bf16 K-major tile
+    static constexpr int LA = 64 * LSTRIDE * 4;              // fp32 [64][LSTRIDE]
     static constexpr int OFF_KQ = 0;
     static constexpr int OFF_V = OFF_KQ + KQ;
-    static constexpr int OFF_L = OFF_V + V;                  // fp32 [64][LSTRIDE] L (and record staging)
-    static constexpr int OFF_XG = OFF_L + 36864;             // X G hi, lo
-    static constexpr int OFF_X = OFF_XG + 2 * TILE128;       // X hi, lo
+    static constexpr int OFF_L = OFF_V + V;                  // L (strictly lower), fp32
+    static constexpr int OFF_XG = OFF_L + 2 * LA;            // [I; A] hi, lo, then X G hi, lo
+    static constexpr int OFF_X = OFF_XG + 2 * TILE128;       // T hi, lo (MN-major), then X hi, lo
     static constexpr int OFF_D = OFF_X + 2 * TILE128;        // fp32 [64][DSTRIDE]: inverses of the diagonal blocks
     static constexpr int OFF_BAR = OFF_D + 64 * DSTRIDE * 4;
     static constexpr int SMEM = OFF_BAR + 64 + 1024;
     // record staging: [W;Q'] hi | lo over XG, X; U | A U over V, L
     static constexpr int OFF_STAGE_WQ = OFF_XG;
     static constexpr int OFF_STAGE_U = OFF_V;
+    static_assert(OFF_XG % 1024 == 0, "operand tiles on 1024-byte boundaries");
     static_assert(2 * 128 * DK * 2 <= 4 * TILE128, "[W;Q'] staging");
-    static_assert(128 * 128 * 4 <= V + 36864, "U | A U staging for d_v <= 128");
+    static_assert(128 * 128 * 4 <= V + 2 * LA, "U | A U staging for d_v <= 128");  // over V and L
     static constexpr uint32_t T_D = 0;                       // KK / QK (64 cols)
     static constexpr uint32_t T_WU = 128;                    // [W | U] (DK + dv cols)
 };
 
 template <int DK>
-__global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_constant__ GdnParams p) {
+__global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_constant__ GdnParams p) {
     using G = PrepCfg<DK>;
     using R = Rec<DK>;
     extern __shared__ uint8_t smem_raw[];
@@ -136,7 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     __shared__ volatile int abort_flag;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int q4 = warp & 3, hf = warp >> 2;
+    const int q4 = warp & 3, cq = warp >> 2;         // TMEM lane quarter, column quarter
     const int row = q4 * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     const int H = p.H, dv = p.dv;
@@ -168,49 +172,55 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     grid_dependents_launch();
     // ---- loads (every global load issued before the shared stores)
     {
-        constexpr int NKQ = 128 * (DK / 8) / kThreads;
-        constexpr int NV = C * (DVP / 8) / kThreads;
+        constexpr int NKQ = 128 * (DK / 8) / kPrepThreads;
+        constexpr int NV = C * (DVP / 8) / kPrepThreads;
         uint4 kq[NKQ], vv[NV];
 #pragma unroll
         for (int u = 0; u < NKQ; ++u) {
-            const int i = tid + u * kThreads;
+            const int i = tid + u * kPrepThreads;
             const int rr = i / (DK / 8), c8 = (i % (DK / 8)) * 8, t = rr & 63;
             kq[u] = t < n ? __ldg(reinterpret_cast<const uint4*>((rr < 64 ? p.k : p.q) + ((tok0 + t) * H + h) * DK + c8))
                           : make_uint4(0, 0, 0, 0);
         }
 #pragma unroll
         for (int u = 0; u < NV; ++u) {
-            const int i = tid + u * kThreads;
+            const int i = tid + u * kPrepThreads;
             const int t = i / (dv / 8), r8 = (i % (dv / 8)) * 8;
             vv[u] = (do_u && i < C * (dv / 8) && t < n) ? __ldg(reinterpret_cast<const uint4*>(p.v + ((tok0 + t) * H + h) * dv + r8))
                                                 : make_uint4(0, 0, 0, 0);
         }
+        // the gates of the chunk (warp 0)
+        float a0 = 1.f, a1 = 1.f, b0 = 0.f, b1 = 0.f;
+        if (tid < 32) {
+            if (tid < n) { a0 = __ldg(p.alpha + (tok0 + tid) * H + h); b0 = __ldg(p.beta + (tok0 + tid) * H + h); }
+            if (tid + 32 < n) { a1 = __ldg(p.alpha + (tok0 + tid + 32) * H + h); b1 = __ldg(p.beta + (tok0 + tid + 32) * H + h); }
+        }
 #pragma unroll
         for (int u = 0; u < NKQ; ++u) {
-            const int i = tid + u * kThreads;
+            const int i = tid + u * kPrepThreads;
             const int rr = i / (DK / 8), c8 = (i % (DK / 8)) * 8;
             V4(oKQ + sw128_off16(rr, c8, 128)) = kq[u];
         }
 #pragma unroll
         for (int u = 0; u < NV; ++u) {
-            const int i = tid + u * kThreads;
+            const int i = tid + u * kPrepThreads;
             if (do_u && i < C * (dv / 8)) V4(oV + sw128_off16(i / (dv / 8), (i % (dv / 8)) * 8, C)) = vv[u];
         }
-    }
-    if (tid < 32) {
-        float x0 = tid < n ? logf(__ldg(p.alpha + (tok0 + tid) * H + h)) : 0.f;
-        float x1 = tid + 32 < n ? logf(__ldg(p.alpha + (tok0 + tid + 32) * H + h)) : 0.f;
+        if (tid < 32) {
+            float x0 = tid < n ? logf(a0) : 0.f;
+            float x1 = tid + 32 < n ? logf(a1) : 0.f;
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const float y0 = __shfl_up_sync(0xffffffffu, x0, o);
-            const float y1 = __shfl_up_sync(0xffffffffu, x1, o);
-            if (tid >= o) { x0 += y0; x1 += y1; }
+            for (int o = 1; o < 32; o <<= 1) {
+                const float y0 = __shfl_up_sync(0xffffffffu, x0, o);
+                const float y1 = __shfl_up_sync(0xffffffffu, x1, o);
+                if (tid >= o) { x0 += y0; x1 += y1; }
+            }
+            x1 += __shfl_sync(0xffffffffu, x0, 31);
+            gs[tid] = x0;
+            gs[tid + 32] = x1;
+            bs[tid] = b0;
+            bs[tid + 32] = b1;
         }
-        x1 += __shfl_sync(0xffffffffu, x0, 31);
-        gs[tid] = x0;
-        gs[tid + 32] = x1;
-        bs[tid] = tid < n ? __ldg(p.beta + (tok0 + tid) * H + h) : 0.f;
-        bs[tid + 32] = tid + 32 < n ? __ldg(p.beta + (tok0 + tid + 32) * H + h) : 0.f;
     }
     fence_proxy_async_smem();
     tc_fence_before();
@@ -253,33 +263,33 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     // ---------------------------------------------------------------- L (rows < 64), A (rows >= 64)
     // L goes to shared memory in fp32 for the solve of T = (I + L)^-1; the
     // rows of [I; A] go straight into the A operand of X = [I; A] T (bf16 hi |
-    // lo, K-major, over the XG tiles)
+    // lo, K-major, over the XG tiles).  Thread (row, cq) forms columns
+    // 16 cq .. 16 cq + 15 of TMEM row `row`.
     if (ok) {
-        // thread (row, hf) handles columns hf*32 .. hf*32+31 of TMEM row `row`
-        uint32_t v[32];
-        tmem_ld32(tmem + lane_off + G::T_D + hf * 32, v);
+        uint32_t v[16];
+        tmem_ld16(tmem + lane_off + G::T_D + cq * 16, v);
         tmem_ld_wait();
         const int t = row & 63;
         const float gt2 = g2[t];
-        float y[32];
+        float y[16];
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-            const int j = hf * 32 + c;
+        for (int c = 0; c < 16; ++c) {
+            const int j = cq * 16 + c;
             const bool keep = (row < 64) ? (j < t) : (j <= t);
             y[c] = (keep && t < n) ? ex2(gt2 - g2[j]) * bs[j] * __uint_as_float(v[c]) : 0.f;
         }
         if (row < 64) {
-            float* dst = Lm + t * LSTRIDE + hf * 32;
+            float* dst = Lm + t * LSTRIDE + cq * 16;
 #pragma unroll
-            for (int j4 = 0; j4 < 32; j4 += 4) *reinterpret_cast<float4*>(dst + j4) = make_float4(y[j4], y[j4 + 1], y[j4 + 2], y[j4 + 3]);
+            for (int j4 = 0; j4 < 16; j4 += 4) *reinterpret_cast<float4*>(dst + j4) = make_float4(y[j4], y[j4 + 1], y[j4 + 2], y[j4 + 3]);
 #pragma unroll
-            for (int c = 0; c < 32; ++c) y[c] = (hf * 32 + c == row) ? 1.f : 0.f;     // row of I
+            for (int c = 0; c < 16; ++c) y[c] = (cq * 16 + c == row) ? 1.f : 0.f;     // row of I
         }
 #pragma unroll
-        for (int j8 = 0; j8 < 32; j8 += 8) {
+        for (int j8 = 0; j8 < 16; j8 += 8) {
             uint4 hi, lo;
             split8(y + j8, hi, lo);
-            const uint32_t off = sw128_off16(row, hf * 32 + j8, 128);
+            const uint32_t off = sw128_off16(row, cq * 16 + j8, 128);
             V4(oXG + off) = hi;
             V4(oXG + T128 + off) = lo;
         }
@@ -307,76 +317,68 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
         for (int i = 0; i < 16; ++i) Dm[(16 * kb + i) * DSTRIDE + c] = d[i];
     }
     __syncthreads();
-    // Four threads per row p (tid = 4p + q); thread q owns columns
-    // 16 k + 4 q .. + 3 of every block k; warps of rows in block top skip the
-    // blocks right of it.  T leaves as the B operand (MN-major, rows = the
-    // contraction index) of X = [I; A] T, bf16 hi | lo over the X tiles.
+    // Eight threads per row pr (tid = 8 pr + q); thread q owns columns
+    // 16 k + 2 q, 16 k + 2 q + 1 of every block k; warps (four rows of one
+    // block) skip the blocks right of it.  T leaves as the B operand
+    // (MN-major, rows = the contraction index) of X = [I; A] T, bf16 hi | lo
+    // over the X tiles.
     if (ok) {
-        const int pr = tid >> 2, q = tid & 3;
-        float xs[16];                                 // xs[4k + e] = x[16k + 4q + e]
+        const int pr = tid >> 3, q = tid & 7;
+        float xs[8];                                  // xs[2k + e] = x[16k + 2q + e]
 #pragma unroll
         for (int k = 0; k < 4; ++k)
 #pragma unroll
-            for (int e = 0; e < 4; ++e) xs[4 * k + e] = (16 * k + 4 * q + e == pr) ? 1.f : 0.f;
-        const int top = pr >> 4;                      // uniform per warp (8 rows of one block)
+            for (int e = 0; e < 2; ++e) xs[2 * k + e] = (16 * k + 2 * q + e == pr) ? 1.f : 0.f;
+        const int top = pr >> 4;                      // uniform per warp (four rows of one block)
 #pragma unroll
         for (int jb = 3; jb >= 0; --jb) {
             if (jb > top) continue;
-            // yv[o][e] = current x[16 jb + 4 (q ^ o) + e]
-            float yv[4][4];
+            // yv[o][e] = current x[16 jb + 2 (q ^ o) + e]
+            float yv[8][2];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float a = xs[4 * jb + e];
+            for (int e = 0; e < 2; ++e) {
+                const float a = xs[2 * jb + e];
                 yv[0][e] = a;
-                yv[1][e] = __shfl_xor_sync(0xffffffffu, a, 1);
-                yv[2][e] = __shfl_xor_sync(0xffffffffu, a, 2);
-                yv[3][e] = __shfl_xor_sync(0xffffffffu, a, 3);
+#pragma unroll
+                for (int o = 1; o < 8; ++o) yv[o][e] = __shfl_xor_sync(0xffffffffu, a, o);
             }
-            float xb[4] = {0.f, 0.f, 0.f, 0.f};
+            float xb[2] = {0.f, 0.f};
 #pragma unroll
-            for (int o = 0; o < 4; ++o)
+            for (int o = 0; o < 8; ++o)
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float4 d4 = *reinterpret_cast<const float4*>(Dm + (16 * jb + 4 * (q ^ o) + e) * DSTRIDE + 4 * q);
-                    xb[0] = fmaf(yv[o][e], d4.x, xb[0]); xb[1] = fmaf(yv[o][e], d4.y, xb[1]);
-                    xb[2] = fmaf(yv[o][e], d4.z, xb[2]); xb[3] = fmaf(yv[o][e], d4.w, xb[3]);
+                for (int e = 0; e < 2; ++e) {
+                    const float2 d2 = *reinterpret_cast<const float2*>(Dm + (16 * jb + 2 * (q ^ o) + e) * DSTRIDE + 2 * q);
+                    xb[0] = fmaf(yv[o][e], d2.x, xb[0]);
+                    xb[1] = fmaf(yv[o][e], d2.y, xb[1]);
                 }
-            float xv[4][4];
+            float xv[8][2];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                xs[4 * jb + c] = xb[c];
+            for (int c = 0; c < 2; ++c) {
+                xs[2 * jb + c] = xb[c];
                 xv[0][c] = xb[c];
-                xv[1][c] = __shfl_xor_sync(0xffffffffu, xb[c], 1);
-                xv[2][c] = __shfl_xor_sync(0xffffffffu, xb[c], 2);
-                xv[3][c] = __shfl_xor_sync(0xffffffffu, xb[c], 3);
+#pragma unroll
+                for (int o = 1; o < 8; ++o) xv[o][c] = __shfl_xor_sync(0xffffffffu, xb[c], o);
             }
 #pragma unroll
             for (int kb = 0; kb < jb; ++kb)
 #pragma unroll
-                for (int o = 0; o < 4; ++o)
+                for (int o = 0; o < 8; ++o)
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float4 l4 = *reinterpret_cast<const float4*>(
-                            Lm + (16 * jb + 4 * (q ^ o) + e) * LSTRIDE + 16 * kb + 4 * q);
-                        xs[4 * kb + 0] = fmaf(-xv[o][e], l4.x, xs[4 * kb + 0]);
-                        xs[4 * kb + 1] = fmaf(-xv[o][e], l4.y, xs[4 * kb + 1]);
-                        xs[4 * kb + 2] = fmaf(-xv[o][e], l4.z, xs[4 * kb + 2]);
-                        xs[4 * kb + 3] = fmaf(-xv[o][e], l4.w, xs[4 * kb + 3]);
+                    for (int e = 0; e < 2; ++e) {
+                        const float2 l2 = *reinterpret_cast<const float2*>(
+                            Lm + (16 * jb + 2 * (q ^ o) + e) * LSTRIDE + 16 * kb + 2 * q);
+                        xs[2 * kb + 0] = fmaf(-xv[o][e], l2.x, xs[2 * kb + 0]);
+                        xs[2 * kb + 1] = fmaf(-xv[o][e], l2.y, xs[2 * kb + 1]);
                     }
         }
-        // T row pr, columns 16 k + 4 q .. + 3: 8 bytes of each of hi and lo
+        // T row pr, columns 16 k + 2 q and + 1: 4 bytes of each of hi and lo
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            float hi4[4], lo4[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const __nv_bfloat16 h = __float2bfloat16_rn(xs[4 * k + e]);
-                hi4[e] = __bfloat162float(h);
-                lo4[e] = xs[4 * k + e] - hi4[e];
-            }
-            const uint32_t off = sw128_off16(pr, 16 * k + 4 * q, 64);
-            *reinterpret_cast<uint2*>(smem + oX + off) = make_uint2(pack_bf16x2(hi4[0], hi4[1]), pack_bf16x2(hi4[2], hi4[3]));
-            *reinterpret_cast<uint2*>(smem + oX + 64 * 128 + off) = make_uint2(pack_bf16x2(lo4[0], lo4[1]), pack_bf16x2(lo4[2], lo4[3]));
+            const __nv_bfloat16 h0 = __float2bfloat16_rn(xs[2 * k]), h1 = __float2bfloat16_rn(xs[2 * k + 1]);
+            const float f0 = __bfloat162float(h0), f1 = __bfloat162float(h1);
+            const uint32_t off = sw128_off16(pr, 16 * k + 2 * q, 64);
+            *reinterpret_cast<uint32_t*>(smem + oX + off) = pack_bf16x2(f0, f1);
+            *reinterpret_cast<uint32_t*>(smem + oX + 64 * 128 + off) = pack_bf16x2(xs[2 * k] - f0, xs[2 * k + 1] - f1);
         }
     }
     fence_proxy_async_smem();
@@ -401,19 +403,19 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     if (ok) ok = mma_wait();
     // operands: X G (for W) and X (for U), K-major rows, from TMEM
     if (ok) {
-        uint32_t v[32];
-        tmem_ld32(tmem + lane_off + G::T_D + hf * 32, v);
+        uint32_t v[16];
+        tmem_ld16(tmem + lane_off + G::T_D + cq * 16, v);
         tmem_ld_wait();
 #pragma unroll
-        for (int j8 = 0; j8 < 32; j8 += 8) {
+        for (int j8 = 0; j8 < 16; j8 += 8) {
             float xr[8], xg[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 xr[e] = __uint_as_float(v[j8 + e]);
-                xg[e] = xr[e] * Gs[hf * 32 + j8 + e];
+                xg[e] = xr[e] * Gs[cq * 16 + j8 + e];
             }
             uint4 hi, lo;
-            const uint32_t off = sw128_off16(row, hf * 32 + j8, 128);
+            const uint32_t off = sw128_off16(row, cq * 16 + j8, 128);
             if (do_w) {
                 split8(xg, hi, lo);
                 V4(oXG + off) = hi;
@@ -452,22 +454,23 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
     if (ok) ok = mma_wait();
     // ---------------------------------------------------------------- record: [W; Q'] image, U | A U
     // Both are staged in shared memory in their record layout (the MMA
-    // operands they overwrite are consumed) and leave in bulk copies.
+    // operands they overwrite are consumed) and leave in bulk copies.  Thread
+    // (row, cq) takes 16-column pieces cq, cq + 4, ...
     if (ok) {
         const int t = row & 63;
         const float gt = Gs[t];
         const uint32_t oWQ = G::OFF_STAGE_WQ;
-        for (int cb = hf * (DK / 2); do_w && cb < (hf + 1) * (DK / 2); cb += 32) {
-            uint32_t v[32];
-            tmem_ld32(tmem + lane_off + G::T_WU + cb, v);
+        for (int cb = 16 * cq; do_w && cb < DK; cb += 64) {
+            uint32_t v[16];
+            tmem_ld16(tmem + lane_off + G::T_WU + cb, v);
             tmem_ld_wait();
-            float y[32];
+            float y[16];
 #pragma unroll
-            for (int j = 0; j < 32; ++j) y[j] = __uint_as_float(v[j]);
+            for (int j = 0; j < 16; ++j) y[j] = __uint_as_float(v[j]);
             if (row >= 64) {
                 // Q' = G Q - A W ; row `row` of [K;Q] holds q_t
 #pragma unroll
-                for (int j8 = 0; j8 < 32; j8 += 8) {
+                for (int j8 = 0; j8 < 16; j8 += 8) {
                     const uint4 q8 = V4(oKQ + sw128_off16(row, cb + j8, 128));
                     const uint32_t* qw = reinterpret_cast<const uint32_t*>(&q8);
 #pragma unroll
@@ -479,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
                 }
             }
 #pragma unroll
-            for (int j8 = 0; j8 < 32; j8 += 8) {
+            for (int j8 = 0; j8 < 16; j8 += 8) {
                 uint4 hi, lo;
                 split8(y + j8, hi, lo);
                 const uint32_t off = sw128_off16(row, cb + j8, 128);
@@ -487,14 +490,13 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_prep_kernel(const __grid_cons
                 V4(oWQ + (uint32_t)R::WQH + off) = lo;
             }
         }
-        const int dh = ((dv / 2) + 31) / 32 * 32;
         float* us = reinterpret_cast<float*>(smem + G::OFF_STAGE_U);
-        for (int rc = hf * dh; do_u && rc < min(dv, (hf + 1) * dh); rc += 32) {
-            uint32_t v[32];
-            tmem_ld32(tmem + lane_off + G::T_WU + DK + rc, v);
+        for (int rc = 16 * cq; do_u && rc < dv; rc += 64) {
+            uint32_t v[16];
+            tmem_ld16(tmem + lane_off + G::T_WU + DK + rc, v);
             tmem_ld_wait();
 #pragma unroll
-            for (int j4 = 0; j4 < 32; j4 += 4)
+            for (int j4 = 0; j4 < 16; j4 += 4)
                 *reinterpret_cast<uint4*>(us + uau_idx(row, rc + j4)) = make_uint4(v[j4], v[j4 + 1], v[j4 + 2], v[j4 + 3]);
         }
     }
@@ -831,7 +833,7 @@ void configure_once(int smem) {
 template <int DK>
 void launch_prep_dk(const GdnParams& p, cudaStream_t s) {
     configure_once<gdn_prep_kernel<DK>>(PrepCfg<DK>::SMEM);
-    launch_pdl(gdn_prep_kernel<DK>, dim3(p.total_chunks * p.H * p.prep_parts), dim3(kThreads), PrepCfg<DK>::SMEM, s, p);
+    launch_pdl(gdn_prep_kernel<DK>, dim3(p.total_chunks * p.H * p.prep_parts), dim3(kPrepThreads), PrepCfg<DK>::SMEM, s, p);
 }
 
 template <int DK, int CW>
