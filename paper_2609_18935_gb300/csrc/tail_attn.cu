@@ -169,9 +169,11 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
 // 2 c0 + 1, or 2 c0 when the tile is also c0's first segment) and the first
 // segments 2 c of the others.  A thread owns four columns of one row (rows
 // fastest across threads, as in the partial layout) and merges the partials
-// online, eight at a time, each batch's (max, sum) pairs and O pieces loaded
+// online, two at a time, each batch's (max, sum) pairs and O pieces loaded
 // together.
-__global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant__ AttnParams p) {
+// At most 36 registers a thread keep seven blocks on an SM, so that the
+// grid of a full round (32 query tiles x 32 blocks) runs in one wave.
+__global__ void __launch_bounds__(256, 7) attn_combine_kernel(const __grid_constant__ AttnParams p) {
     grid_dependency_wait();
     grid_dependents_launch();
     const int cb = p.split_cb[blockIdx.x];
@@ -181,7 +183,6 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
     while (c1 + 1 < p.n_ctas && p.cta_tile[c1 + 1] == t && p.cta_k[c1 + 1] > 0) ++c1;
     const int slot0 = (p.cta_tile[c0] == t) ? 2 * c0 : 2 * c0 + 1;
     const int n_parts = c1 - c0 + 1;
-    auto slot_of = [&](int q) -> int64_t { return q == 0 ? slot0 : 2 * (c0 + q); };
 
     int lo = 0, hi = p.n_chars - 1;                                // last b with tile_off <= t
     while (lo < hi) {
@@ -192,7 +193,6 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
     const int local = t - c.tile_off;
     const int kvh = local / c.n_qtiles, qt = local % c.n_qtiles;
     const int D = p.D;
-    const int groups = D / 32;                                     // 32-column groups
     const int item = blockIdx.y * blockDim.x + threadIdx.x;        // (4-column piece, row): rows fastest
     const int r = item % kRows;
     const int piece = item / kRows;
@@ -200,7 +200,12 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
     const int cg = piece >> 3, q4 = piece & 7;
     const int tok = qt * p.tok_per_tile + r / p.g;
     if (tok >= c.M) return;
-    constexpr int kBatch = 8;
+    __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + kvh * p.g + (r % p.g)) * D + cg * 32 + q4 * 4;
+    // this thread's piece of slot s: po + s * D * kRows floats; its (max, sum): pm + s * 2 kRows
+    const float* po = p.part_o + ((cg * 8 + q4) * kRows + r) * 4;
+    const float* pm = p.part_ml + r * 2;
+    const int sstride = D * kRows;
+    constexpr int kBatch = 2;
     float mx = -INFINITY, den = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int q0 = 0; q0 < n_parts; q0 += kBatch) {
@@ -209,9 +214,9 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
 #pragma unroll
         for (int u = 0; u < kBatch; ++u) {
             if (q0 + u < n_parts) {
-                const int64_t slot = slot_of(q0 + u);
-                ml[u] = *reinterpret_cast<const float2*>(p.part_ml + (slot * kRows + r) * 2);
-                x[u] = *reinterpret_cast<const float4*>(p.part_o + (((slot * groups + cg) * 8 + q4) * kRows + r) * 4);
+                const int slot = (q0 + u == 0) ? slot0 : 2 * (c0 + q0 + u);
+                ml[u] = *reinterpret_cast<const float2*>(pm + slot * (2 * kRows));
+                x[u] = *reinterpret_cast<const float4*>(po + slot * sstride);
             } else {
                 ml[u] = make_float2(-INFINITY, 0.f);
             }
@@ -234,8 +239,6 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
         mx = nmx;
     }
     const float inv = den > 0.f ? 1.f / den : 0.f;
-    const int hq = kvh * p.g + (r % p.g);
-    __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + hq) * D + cg * 32 + q4 * 4;
     *reinterpret_cast<uint2*>(o) = make_uint2(f2_to_bf2(acc.x * inv, acc.y * inv), f2_to_bf2(acc.z * inv, acc.w * inv));
 }
 
