@@ -324,7 +324,7 @@ def run_kvm(args):
         tot = int(tail_cu[-1])
         d_out = {l: torch.empty((tot, s.n_q_heads, s.head_dim) if k == W.ATTN else (tot, s.n_gdn_heads, s.d_v),
                                 dtype=torch.bfloat16, device="cuda") for l, k in enumerate(s.layer_kind)}
-        h_in = {l: {k: v.cpu().pin_memory() for k, v in x.items()} for l, x in d_in.items()}
+        h_in = kvm.pinned_layer_inputs(d_in)              # one pinned arena per layer
         h_out = {l: torch.empty(o.shape, dtype=o.dtype).pin_memory() for l, o in d_out.items()}
         rounds.append(dict(cu=cu, sb=sb, se=se, tails=tails, tail_cu=tail_cu, d_in=d_in, d_out=d_out,
                            h_in=h_in, h_out=h_out))

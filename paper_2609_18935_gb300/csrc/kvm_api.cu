@@ -882,19 +882,45 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
         n[3] = n[4] = attn ? 0 : (size_t)total * c->H * 4;
         n[5] = (size_t)total * (attn ? c->Hq * c->D : c->H * c->dv) * 2;
     };
+    // Host-resident rounds stage a layer's inputs q, k, v, alpha, beta back to
+    // back from the layer's staging base (each piece rounded up to 16 bytes).
+    // Pieces that also lie back to back in the caller's memory go up in one
+    // copy: a copy costs ~5 us before its first byte, so a caller that keeps
+    // a layer's inputs in one pinned arena pays that once per layer.
+    auto stage_in = [&](int l, size_t off[5]) {
+        size_t n[6];
+        sizes(l, n);
+        size_t o = c->stage_in_off[5 * l];
+        for (int i = 0; i < 5; ++i) {
+            off[i] = o;
+            o += (n[i] + 15) / 16 * 16;
+        }
+    };
     if (host_io) {
         // every layer's inputs go up on the copy stream at once (after the work
         // already queued on s, which may still read the staging buffers)
         CUDA_TRY(cudaEventRecord(c->ev_start, s));
         CUDA_TRY(cudaStreamWaitEvent(c->copy_stream, c->ev_start, 0));
         for (int l = 0; l < c->n_layers; ++l) {
-            size_t n[6];
+            size_t n[6], off[5];
             sizes(l, n);
-            const void* src[5] = {r->q[l], r->k[l], r->v[l], r->alpha ? r->alpha[l] : nullptr,
-                                  r->beta ? r->beta[l] : nullptr};
-            for (int i = 0; i < 5; ++i)
-                if (n[i]) CUDA_TRY(cudaMemcpyAsync(c->stage + c->stage_in_off[5 * l + i], src[i], n[i],
-                                                   cudaMemcpyHostToDevice, c->copy_stream));
+            stage_in(l, off);
+            const char* src[5] = {static_cast<const char*>(r->q[l]), static_cast<const char*>(r->k[l]),
+                                  static_cast<const char*>(r->v[l]),
+                                  r->alpha ? reinterpret_cast<const char*>(r->alpha[l]) : nullptr,
+                                  r->beta ? reinterpret_cast<const char*>(r->beta[l]) : nullptr};
+            for (int i = 0; i < 5;) {
+                if (!n[i]) { ++i; continue; }
+                // extend the run while the next piece follows in both places
+                int j = i;
+                size_t bytes = n[i];
+                while (j + 1 < 5 && n[j + 1] && n[j] % 16 == 0 && src[j + 1] == src[j] + n[j]) {
+                    ++j;
+                    bytes += n[j];
+                }
+                CUDA_TRY(cudaMemcpyAsync(c->stage + off[i], src[i], bytes, cudaMemcpyHostToDevice, c->copy_stream));
+                i = j + 1;
+            }
             CUDA_TRY(cudaEventRecord(c->ev_in[l], c->copy_stream));
         }
     }
@@ -932,7 +958,8 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
         void* out = r->out[l];
         if (host_io) {
             CUDA_TRY(cudaStreamWaitEvent(s, c->ev_in[l], 0));
-            const size_t* o = &c->stage_in_off[5 * l];
+            size_t o[5];
+            stage_in(l, o);
             q = c->stage + o[0]; k = c->stage + o[1]; v = c->stage + o[2];
             if (!attn) {
                 al = reinterpret_cast<const float*>(c->stage + o[3]);

@@ -155,6 +155,32 @@ def kv_compact_noalloc(K, V, positions, live, span_begin, span_end, stream=None)
     return new_live.value
 
 
+def pinned_layer_inputs(inputs):
+    """Copy per-layer inputs into one pinned host arena per layer.
+
+    inputs[layer] = dict(q, k, v[, alpha, beta]) (CPU or CUDA tensors).
+    Returns the same structure with views into a pinned arena per layer,
+    laid out q, k, v, alpha, beta back to back (each piece padded to 16
+    bytes), which lets a host-resident update_round move a layer's inputs in
+    one copy."""
+    import torch
+    out = {}
+    for layer, x in inputs.items():
+        keys = [k for k in ("q", "k", "v", "alpha", "beta") if x.get(k) is not None]
+        sizes = [x[k].numel() * x[k].element_size() for k in keys]
+        padded = [(n + 15) // 16 * 16 for n in sizes]
+        arena = torch.empty(sum(padded), dtype=torch.uint8).pin_memory()
+        views, off = {}, 0
+        for k, n, pn in zip(keys, sizes, padded):
+            t = x[k]
+            v = arena[off:off + n].view(t.dtype).view(t.shape)
+            v.copy_(t.cpu())
+            views[k] = v
+            off += pn
+        out[layer] = views
+    return out
+
+
 class Context:
     """A population of character states on the current CUDA device (kvm_create)."""
 

@@ -182,10 +182,13 @@ def test_spans_from_positions():
         pair.ctx.spans_from_positions(0, [0], [10])     # covers no live entry
 
 
-def test_host_resident_round_equals_device_round():
+@pytest.mark.parametrize("arena", [False, True])
+def test_host_resident_round_equals_device_round(arena):
     """kvm_update_round with host-resident (pinned) inputs and outputs runs
     the same kernels as with device tensors: outputs, caches and states
-    bit-identical, over two chained rounds of a 2-character population."""
+    bit-identical, over two chained rounds of a 2-character population.
+    With `arena`, each layer's inputs sit back to back in one pinned buffer
+    and go up in one copy."""
     import torch
     from paper_2609_18935_gb300 import kvm
     shape = W.ModelShape([W.GDN, W.ATTN, W.GDN, W.ATTN], 8, 2, 128, 64, 1e4, 4, 64, 96)
@@ -212,7 +215,8 @@ def test_host_resident_round_equals_device_round():
         tail_cu = np.concatenate([[0], np.cumsum(tails)]).astype(np.int32)
         T = int(tail_cu[-1])
         d_in = W.device_round_inputs(w, 100 + r, tails)
-        h_in = {l: {k: t.cpu().pin_memory() for k, t in x.items()} for l, x in d_in.items()}
+        h_in = (kvm.pinned_layer_inputs(d_in) if arena
+                else {l: {k: t.cpu().pin_memory() for k, t in x.items()} for l, x in d_in.items()})
         shp = lambda l: (T, shape.n_q_heads, shape.head_dim) if shape.layer_kind[l] == W.ATTN else (T, shape.n_gdn_heads, shape.d_v)
         d_out = {l: torch.empty(shp(l), dtype=torch.bfloat16, device="cuda") for l in range(len(shape.layer_kind))}
         h_out = {l: torch.empty(shp(l), dtype=torch.bfloat16).pin_memory() for l in range(len(shape.layer_kind))}
