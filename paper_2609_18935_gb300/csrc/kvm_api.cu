@@ -516,24 +516,21 @@ extern "C" kvm_status kvm_spans_from_positions(kvm_ctx* c, int32_t b, int32_t n,
 // ============================================================================
 namespace {
 
-kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, const int32_t* send,
-                      int32_t* gather_out, cudaStream_t s) {
-    SpanPlan pl;
-    kvm_status st = plan_spans(c, span_cu, sbeg, send, pl);
-    if (st) return st;
-
-    if (c->n_attn > 0) {
+// Compaction of the attention layers [a_lo, a_hi) (K and V slabs of those
+// layers, and the position slab when with_pos) under a validated plan.
+kvm_status launch_compaction(kvm_ctx* c, const SpanPlan& pl, cudaStream_t s, int a_lo, int a_hi, bool with_pos) {
+    if (c->n_attn > 0 && a_hi > a_lo) {
         thread_local static CompactParams p;   // large parameter block, copied into the launch
         std::memset(&p, 0, sizeof p);
         p.n_chars = c->B;
-        p.n_kv_slabs = 2 * c->n_attn * c->Hkv;
+        p.n_kv_slabs = 2 * (a_hi - a_lo) * c->Hkv;
         p.vec_per_row = c->D * 2 / 16;
         p.rows_kv = c->rows_kv;
         p.rows_pos = c->rows_pos;
         p.epoch = ++c->epoch;
         p.slab_rows = c->T_cap;
-        p.K = reinterpret_cast<uint4*>(c->K);
-        p.V = reinterpret_cast<uint4*>(c->V);
+        p.K = reinterpret_cast<uint4*>(c->K + (size_t)a_lo * c->Hkv * c->T_cap * c->D);
+        p.V = reinterpret_cast<uint4*>(c->V + (size_t)a_lo * c->Hkv * c->T_cap * c->D);
         p.pos = c->pos;
         p.tickets = c->tickets;
         p.flags = c->flags;
@@ -549,7 +546,7 @@ kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, c
             ch.n_seg = pl.n_seg[b];
             ch.cap_off = c->cap_off[b];
             ch.chunks_kv = (moved + p.rows_kv - 1) / p.rows_kv;
-            ch.chunks_pos = (moved + p.rows_pos - 1) / p.rows_pos;
+            ch.chunks_pos = with_pos ? (moved + p.rows_pos - 1) / p.rows_pos : 0;
             ch.blk_off = blk;
             ch.flag_off = c->flag_off[b];
             blk += p.n_kv_slabs * ch.chunks_kv + ch.chunks_pos;
@@ -564,6 +561,11 @@ kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, c
             LAUNCH_CHECK(c);
         }
     }
+    return KVM_OK;
+}
+
+// The optional gather map (new slot -> old slot) of a validated plan.
+kvm_status launch_gather(kvm_ctx* c, const SpanPlan& pl, int32_t* gather_out, cudaStream_t s) {
     if (gather_out) {
         thread_local static GatherParams gp;
         std::memset(&gp, 0, sizeof gp);
@@ -588,6 +590,11 @@ kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, c
             LAUNCH_CHECK(c);
         }
     }
+    return KVM_OK;
+}
+
+// Host bookkeeping of a validated plan: live lengths and the position mirror.
+void apply_plan(kvm_ctx* c, const SpanPlan& pl, const int32_t* span_cu, const int32_t* sbeg, const int32_t* send) {
     // host bookkeeping: live lengths and the position mirror
     for (int b = 0; b < c->B; ++b) {
         if (pl.n_seg[b] == 0) continue;
@@ -603,6 +610,19 @@ kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, c
         P.swap(keep);
         c->live[b] = pl.L_new[b];
     }
+}
+
+
+kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, const int32_t* send,
+                      int32_t* gather_out, cudaStream_t s) {
+    SpanPlan pl;
+    kvm_status st = plan_spans(c, span_cu, sbeg, send, pl);
+    if (st) return st;
+    st = launch_compaction(c, pl, s, 0, c->n_attn, true);
+    if (st) return st;
+    st = launch_gather(c, pl, gather_out, s);
+    if (st) return st;
+    apply_plan(c, pl, span_cu, sbeg, send);
     return KVM_OK;
 }
 
@@ -924,26 +944,36 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
             CUDA_TRY(cudaEventRecord(c->ev_in[l], c->copy_stream));
         }
     }
-    // Compaction changes only the attention layers' caches.  With recurrent
-    // layers ahead of the first attention layer it runs on the compaction
+    // Compaction changes only the attention layers' caches.  When recurrent
+    // layers come before the first attention layer, it runs on the compaction
     // stream beside them (after everything already queued on s), and s joins
-    // it one layer early, so the join never stalls the stream and breaks the
-    // launch overlap of a kernel that waits anyway.
+    // it one layer before the first attention layer, so the join never stalls
+    // and breaks the launch overlap of a kernel that waits anyway.  (One
+    // launch for all attention layers: launches per layer have too few blocks
+    // each and slow the recurrent layers they run beside.)
     int first_attn = c->n_layers;
     for (int l = c->n_layers - 1; l >= 0; --l)
         if (c->kind[l] == KVM_LAYER_ATTN) first_attn = l;
     const bool side = first_attn > 0 && first_attn < c->n_layers;
-    const int join_at = first_attn >= 2 ? first_attn - 1 : first_attn;
-    if (side) {
-        CUDA_TRY(cudaEventRecord(c->ev_round, s));
-        CUDA_TRY(cudaStreamWaitEvent(c->compact_stream, c->ev_round, 0));
-        st = do_compact(c, r->span_cu, r->span_begin, r->span_end, r->gather_out, c->compact_stream);
+    {
+        SpanPlan pl;
+        st = plan_spans(c, r->span_cu, r->span_begin, r->span_end, pl);
         if (st) return st;
-        CUDA_TRY(cudaEventRecord(c->ev_compacted, c->compact_stream));
-    } else {
-        st = do_compact(c, r->span_cu, r->span_begin, r->span_end, r->gather_out, s);
+        cudaStream_t cs = side ? c->compact_stream : s;
+        if (side) {
+            CUDA_TRY(cudaEventRecord(c->ev_round, s));
+            CUDA_TRY(cudaStreamWaitEvent(cs, c->ev_round, 0));
+        }
+        // the gather map depends on the plan only; it goes first so that the
+        // events of the compactions cover it
+        st = launch_gather(c, pl, r->gather_out, cs);
         if (st) return st;
+        st = launch_compaction(c, pl, cs, 0, c->n_attn, true);
+        if (st) return st;
+        if (side) CUDA_TRY(cudaEventRecord(c->ev_compacted, cs));
+        apply_plan(c, pl, r->span_cu, r->span_begin, r->span_end);
     }
+    const int join_at = first_attn >= 2 ? first_attn - 1 : first_attn;
     bool joined = !side;
     auto join = [&]() -> cudaError_t {
         if (joined) return cudaSuccess;
