@@ -189,13 +189,24 @@ kvm_status kvm_gdn_chunk_scan_from_state(kvm_ctx* ctx, int32_t layer, const int3
  * layers).  tail_cu host [n_chars+1]. */
 kvm_status kvm_advance(kvm_ctx* ctx, const int32_t* tail_cu);
 
-/* One whole maintenance round: kv_compact, then every layer in model order
- * (tail_attn_prefill or gdn_chunk_scan_from_state), then advance.
- * Per-layer arrays are indexed by model layer; alpha/beta entries of
- * attention layers are ignored.  io_on_host = 0: q/k/v/alpha/beta/out are
- * device pointers.  io_on_host = 1: they are host pointers (pinned memory
- * for asynchronous copies); the library copies each layer's inputs into its
- * own device staging buffers and the layer's output back, on `stream`. */
+/* One whole maintenance round (Eq. 2 then Eq. 3 for every layer; §4.1, §4.2):
+ * kv_compact, then every layer in model order (tail_attn_prefill or
+ * gdn_chunk_scan_from_state), then advance.  Per-layer arrays are indexed by
+ * model layer; alpha/beta entries of attention layers are ignored.
+ * Ordering: everything the round does is complete when the work enqueued on
+ * `stream` up to this call's return has completed.  Internally the
+ * compaction may run on a stream of the context beside the recurrent layers
+ * that precede the first attention layer (it touches only the attention
+ * caches), joined back into `stream` before the first attention layer.
+ * io_on_host = 0: q/k/v/alpha/beta/out are device pointers.
+ * io_on_host = 1: they are host pointers (pinned memory for asynchronous
+ * copies, valid until `stream` has completed the round); the library copies
+ * every layer's inputs up into its own device staging buffers on a copy
+ * stream at once, each layer waiting only for its own, and each layer's
+ * output back while the next layers compute.  Inputs of one layer that lie
+ * back to back in host memory (q, k, v, alpha, beta in that order, each
+ * padded to 16 bytes) go up in one copy.  Errors: as the per-layer calls,
+ * all detected on the host before the first launch. */
 typedef struct kvm_round {
     const int32_t* span_cu;        /* host [n_chars+1] */
     const int32_t* span_begin;     /* host */
