@@ -12,7 +12,9 @@
 //   E  = U - W S0^T,   O = A U + Q' S0^T               (= G Q S0^T + A E)
 //   S^T = G_C S0^T + K^T diag(w) E
 // Everything above the line "E = ..." is independent of the state, so it runs
-// in a prep kernel with one block per (chunk, head), all chunks in parallel;
+// in a prep kernel with one block of 512 threads per (chunk, head) (two when
+// both fit on the SMs: one writes [W; Q'] and K, the other U | A U), all
+// chunks in parallel;
 // it leaves per (chunk, head) a record with [W; Q'] and K as ready-made MMA
 // operand images, U and A U in fp32, w and G_C.  The scan kernel then walks
 // the chunks of each (character, head, d_v slice) in order with the state in

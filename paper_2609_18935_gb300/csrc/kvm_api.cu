@@ -109,7 +109,7 @@ struct kvm_ctx {
     cudaEvent_t ev_round = nullptr, ev_compacted = nullptr;
     std::vector<cudaEvent_t> ev_in, ev_done;   // per layer: inputs landed, outputs written
     double inv_freq[kMaxRotaryHalf] = {};
-    CUtensorMap tmap_q, tmap_k, tmap_v;   // TMA maps of q_rot, K, V (attention layers only)
+    CUtensorMap tmap_k, tmap_v;           // TMA maps of K, V (attention layers only)
     int64_t launches = 0;
     int rows_kv = 0, rows_pos = 0;
     // per-kernel timing (kvm_profile_*)
@@ -354,14 +354,10 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         // TMA maps: rotated q as [max_tail][Hq][D] with a (64, g, 128/g) box;
         // every layer's K and V as rows of D with a (64, 64) box
         const uint64_t row_bytes = (uint64_t)c->D * 2;
-        const uint64_t qd[3] = {(uint64_t)c->D, (uint64_t)c->Hq, (uint64_t)max_tail_tokens};
-        const uint64_t qs[2] = {row_bytes, row_bytes * c->Hq};
-        const uint32_t qb[3] = {64, (uint32_t)c->g, (uint32_t)(kAttnRows / c->g)};
         const uint64_t kd[2] = {(uint64_t)c->D, (uint64_t)c->n_attn * c->Hkv * c->T_cap};
         const uint64_t ks[1] = {row_bytes};
         const uint32_t kb[2] = {64, 64};
         if (kd[1] > (uint64_t)INT32_MAX ||
-            !encode_bf16_sw128(&c->tmap_q, c->q_rot, 3, qd, qs, qb) ||
             !encode_bf16_sw128(&c->tmap_k, c->K, 2, kd, ks, kb) ||
             !encode_bf16_sw128(&c->tmap_v, c->V, 2, kd, ks, kb)) {
             free_all(c);
@@ -646,7 +642,6 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
     thread_local static AttnParams p;
     std::memset(&p, 0, sizeof p);
     const int a = c->attn_idx[layer];
-    p.tmap_q = c->tmap_q;
     p.tmap_k = c->tmap_k;
     p.tmap_v = c->tmap_v;
     p.attn_layer = a;

@@ -118,9 +118,7 @@ struct AttnChar {
 constexpr int kMaxAttnCtas = 320;
 
 struct AttnParams {
-    // TMA maps: rotated q [max_tail][Hq][D] (box 64 x g x 128/g), and every
-    // layer's K / V slabs as rows of D (box 64 x 64), 128-byte swizzle
-    CUtensorMap tmap_q;
+    // TMA maps: every layer's K / V slabs as rows of D (box 64 x 64), 128-byte swizzle
     CUtensorMap tmap_k;
     CUtensorMap tmap_v;
     int32_t attn_layer;   // index among attention layers
