@@ -260,6 +260,13 @@ __global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_
                      idesc_bf16_f32(128, C, false), ks > 0);
         }
         mma_commit(mbar);
+        if (do_w) {
+            // the K image (rows 0..63 of each 64-column region of [K;Q]) is
+            // final already; it leaves now, beside the rest of the kernel
+            for (int r = 0; r < DK / 64; ++r)
+                bulk_store(rec + 2 * R::WQH + r * (64 * 128), sb + oKQ + r * (128 * 128), 64 * 128);
+            bulk_commit();
+        }
     }
     ok = mma_wait();                                // also publishes Gs
     // ---------------------------------------------------------------- L (rows < 64), A (rows >= 64)
@@ -456,67 +463,81 @@ __global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_
     if (ok) ok = mma_wait();
     // ---------------------------------------------------------------- record: [W; Q'] image, U | A U
     // Both are staged in shared memory in their record layout (the MMA
-    // operands they overwrite are consumed) and leave in bulk copies.  Thread
-    // (row, cq) takes 16-column pieces cq, cq + 4, ...
-    if (ok) {
+    // operands they overwrite are consumed), 64 columns at a time: thread
+    // (row, cq) takes the 16-column piece cq of each, and each 64-column
+    // piece leaves in bulk copies while the next one is staged ([W; Q'] keeps
+    // 64-column regions, U | A U 32-column slices, so a piece is contiguous).
+    {
         const int t = row & 63;
         const float gt = Gs[t];
         const uint32_t oWQ = G::OFF_STAGE_WQ;
-        for (int cb = 16 * cq; do_w && cb < DK; cb += 64) {
-            uint32_t v[16];
-            tmem_ld16(tmem + lane_off + G::T_WU + cb, v);
-            tmem_ld_wait();
-            float y[16];
+        float* us = reinterpret_cast<float*>(smem + G::OFF_STAGE_U);
+        const int n_w = do_w ? DK / 64 : 0;
+        const int n_u = do_u ? (dv + 63) / 64 : 0;
+        for (int k = 0; k < n_w + n_u; ++k) {            // uniform per block
+            const bool w_piece = k < n_w;
+            if (ok && w_piece) {
+                const int cb = 64 * k + 16 * cq;
+                uint32_t v[16];
+                tmem_ld16(tmem + lane_off + G::T_WU + cb, v);
+                tmem_ld_wait();
+                float y[16];
 #pragma unroll
-            for (int j = 0; j < 16; ++j) y[j] = __uint_as_float(v[j]);
-            if (row >= 64) {
-                // Q' = G Q - A W ; row `row` of [K;Q] holds q_t
+                for (int j = 0; j < 16; ++j) y[j] = __uint_as_float(v[j]);
+                if (row >= 64) {
+                    // Q' = G Q - A W ; row `row` of [K;Q] holds q_t
 #pragma unroll
-                for (int j8 = 0; j8 < 16; j8 += 8) {
-                    const uint4 q8 = V4(oKQ + sw128_off16(row, cb + j8, 128));
-                    const uint32_t* qw = reinterpret_cast<const uint32_t*>(&q8);
+                    for (int j8 = 0; j8 < 16; j8 += 8) {
+                        const uint4 q8 = V4(oKQ + sw128_off16(row, cb + j8, 128));
+                        const uint32_t* qw = reinterpret_cast<const uint32_t*>(&q8);
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
-                        y[j8 + 2 * e] = gt * f.x - y[j8 + 2 * e];
-                        y[j8 + 2 * e + 1] = gt * f.y - y[j8 + 2 * e + 1];
+                        for (int e = 0; e < 4; ++e) {
+                            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
+                            y[j8 + 2 * e] = gt * f.x - y[j8 + 2 * e];
+                            y[j8 + 2 * e + 1] = gt * f.y - y[j8 + 2 * e + 1];
+                        }
                     }
                 }
-            }
 #pragma unroll
-            for (int j8 = 0; j8 < 16; j8 += 8) {
-                uint4 hi, lo;
-                split8(y + j8, hi, lo);
-                const uint32_t off = sw128_off16(row, cb + j8, 128);
-                V4(oWQ + off) = hi;
-                V4(oWQ + (uint32_t)R::WQH + off) = lo;
+                for (int j8 = 0; j8 < 16; j8 += 8) {
+                    uint4 hi, lo;
+                    split8(y + j8, hi, lo);
+                    const uint32_t off = sw128_off16(row, cb + j8, 128);
+                    V4(oWQ + off) = hi;
+                    V4(oWQ + (uint32_t)R::WQH + off) = lo;
+                }
+            } else if (ok) {
+                const int rc = 64 * (k - n_w) + 16 * cq;
+                if (rc < dv) {                           // uniform per warp
+                    uint32_t v[16];
+                    tmem_ld16(tmem + lane_off + G::T_WU + DK + rc, v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j4 = 0; j4 < 16; j4 += 4)
+                        *reinterpret_cast<uint4*>(us + uau_idx(row, rc + j4)) = make_uint4(v[j4], v[j4 + 1], v[j4 + 2], v[j4 + 3]);
+                }
+            }
+            fence_proxy_async_smem();
+            __syncthreads();
+            if (ok && tid == 0) {
+                if (w_piece) {
+                    bulk_store(rec + k * (128 * 128), sb + oWQ + k * (128 * 128), 128 * 128);
+                    bulk_store(rec + R::WQH + k * (128 * 128), sb + oWQ + (uint32_t)R::WQH + k * (128 * 128), 128 * 128);
+                } else {
+                    const int u = k - n_w;                 // slices 2u, 2u + 1
+                    const int slices = min(2, dv / 32 - 2 * u);
+                    bulk_store(rec + R::uau_off() + (int64_t)u * 2 * (128 * 32 * 4),
+                               sb + G::OFF_STAGE_U + u * 2 * (128 * 32 * 4), slices * (128 * 32 * 4));
+                }
+                bulk_commit();
             }
         }
-        float* us = reinterpret_cast<float*>(smem + G::OFF_STAGE_U);
-        for (int rc = 16 * cq; do_u && rc < dv; rc += 64) {
-            uint32_t v[16];
-            tmem_ld16(tmem + lane_off + G::T_WU + DK + rc, v);
-            tmem_ld_wait();
-#pragma unroll
-            for (int j4 = 0; j4 < 16; j4 += 4)
-                *reinterpret_cast<uint4*>(us + uau_idx(row, rc + j4)) = make_uint4(v[j4], v[j4 + 1], v[j4 + 2], v[j4 + 3]);
+        if (tid == 0) {
+            // the sources must be read before the block's shared memory is
+            // released; the writes complete with the grid, before the scan
+            // (which waits on this grid) reads them
+            bulk_wait_read();
         }
-    }
-    fence_proxy_async_smem();
-    __syncthreads();
-    if (ok && tid == 0) {
-        if (do_w) {
-            bulk_store(rec, sb + G::OFF_STAGE_WQ, 2 * (uint32_t)R::WQH);
-            // K image: rows 0..63 of each 64-column region of [K;Q]
-            for (int r = 0; r < DK / 64; ++r)
-                bulk_store(rec + 2 * R::WQH + r * (64 * 128), sb + oKQ + r * (128 * 128), 64 * 128);
-        }
-        if (do_u) bulk_store(rec + R::uau_off(), sb + G::OFF_STAGE_U, 128u * dv * 4u);
-        bulk_commit();
-        // the sources must be read before the block's shared memory is
-        // released; the writes complete with the grid, before the scan
-        // (which waits on this grid) reads them
-        bulk_wait_read();
     }
     tc_fence_before();
     __syncthreads();
