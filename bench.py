@@ -398,16 +398,16 @@ def run_kvm(args):
         work.profile_enable(False)
         launches = work.launch_count() - launches0
         total_ms = max_over_ranks(float(sum(ms)), world, device="cuda")
-        return total_ms, [r for _, _, r in evs], kernels, launches, (t0, t1)
+        return total_ms, [r for _, _, r in evs], kernels, launches, (t0, t1), ms
 
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    total_ms, rids, _, launches, (t0, t1) = timed(host_io=False)
+    total_ms, rids, _, launches, (t0, t1), _ = timed(host_io=False)
     clk = clocks.summary(t0, t1)
     # per-kernel durations: the same steps again with per-launch events
-    prof_ms, _, kernels, _, _ = timed(host_io=False, profile=True)
-    e2e_ms, e2e_rids, _, _, _ = timed(host_io=True)
+    prof_ms, _, kernels, _, _, _ = timed(host_io=False, profile=True)
+    e2e_ms, e2e_rids, _, _, _, e2e_steps = timed(host_io=True)
     clocks.stop()
 
     toks_rank = sum(sum(rounds[r]["tails"]) for r in rids)
@@ -496,7 +496,10 @@ def run_kvm(args):
         "e2e": {"value": e2e_value, "unit": UNIT,
                 "h2d_bytes_per_step": int(np.mean([rounds[r]["h2d"] for r in e2e_rids])),
                 "d2h_bytes_per_step": int(np.mean([rounds[r]["d2h"] for r in e2e_rids])),
-                "ms_per_step": e2e_ms / args.steps},
+                "ms_per_step": e2e_ms / args.steps,
+                # the host link is shared with the node's other jobs: the
+                # spread of the steps shows whether one of them stalled
+                "ms_per_step_median": float(np.median(e2e_steps)), "ms_per_step_max": float(np.max(e2e_steps))},
         "gpu_launches": launches,
         "kernels": per_kernel,
         "kernel_timing": ("per-launch CUDA events in a second pass over the same steps (events between "
