@@ -43,8 +43,9 @@ class Pair:
         from paper_2609_18935_gb300 import kvm
         self.shape = shape
         s = shape
-        self.ctx = kvm.Context(s.layer_kind, s.n_q_heads, s.n_kv_heads, s.head_dim, s.rotary_dim,
-                               s.rope_theta, s.n_gdn_heads, s.d_k, s.d_v, capacity, max_tail)
+        self._new_ctx = lambda: kvm.Context(s.layer_kind, s.n_q_heads, s.n_kv_heads, s.head_dim, s.rotary_dim,
+                                            s.rope_theta, s.n_gdn_heads, s.d_k, s.d_v, capacity, max_tail)
+        self.ctx = self._new_ctx()
         self.B = len(prefix_len)
         self.oracle = []
         w = W.Workload("custom", seed_index, shape, list(prefix_len), 1)
@@ -90,6 +91,18 @@ class Pair:
                 k, v = self.ctx.get_kv(l, b)
                 snap[(l, b)] = (torch_bf16_bits(k), torch_bf16_bits(v), self.ctx.get_positions(b).cpu().numpy())
         return snap
+
+    def fork(self) -> "Pair":
+        """A second pair holding the same state: a new GPU context filled by
+        kvm_fork from this one and a copy of the oracle states (a per-task
+        root branching from a maintained one, §4.2)."""
+        import copy
+        other = object.__new__(Pair)
+        other.__dict__.update(self.__dict__)
+        other.ctx = self._new_ctx()
+        other.ctx.fork_from(self.ctx)
+        other.oracle = copy.deepcopy(self.oracle)
+        return other
 
     def run_round(self, span_cu, sb, se, tails, inputs, check_bitexact=True, via="update_round"):
         """One round on both sides.  Returns dict of rel-L2 errors and raises on

@@ -127,6 +127,31 @@ def test_many_ragged_tiles_without_key_splits(head_dim):
     _assert_errs(errs, what=f"ragged tiles D={head_dim}")
 
 
+def test_decode_after_maintenance_and_forked_roots():
+    """After a maintenance round, one-token rounds (no removals, one tail
+    token per character: decode steps) continue from the maintained state.
+    A root forked after the maintenance (kvm_fork) decodes other tokens on its
+    own and matches its own copy of the oracle state, while the original
+    keeps matching its own."""
+    from harness import Pair
+    shape = W.npc_shape(4)
+    N = [700, 1100]
+    steps = 3
+    w = W.Workload("decode", 23, shape, N, 1 + 2 * steps)
+    w.plan = [[(0.05, 2, 80), (0.03, 1, 64)]] + [[(0.0, 0, 1), (0.0, 0, 1)]] * (2 * steps)
+    pair = Pair(shape, N, w.capacity(), 80 + 64, seed_index=w.index)
+    live = [pair.ctx.get_live(b)[0] for b in range(2)]
+    span_cu, sb, se, tails = W.round_plan(w, 0, live)
+    _assert_errs(pair.run_round(span_cu, sb, se, tails, W.tail_inputs(w, 0, tails)), what="maintenance")
+    task = pair.fork()
+    for i in range(steps):
+        for p, rnd in ((pair, 1 + i), (task, 1 + steps + i)):      # different tokens on each root
+            live = [p.ctx.get_live(b)[0] for b in range(2)]
+            span_cu, sb, se, tails = W.round_plan(w, rnd, live)
+            assert len(sb) == 0 and tails == [1, 1]
+            _assert_errs(p.run_round(span_cu, sb, se, tails, W.tail_inputs(w, rnd, tails)), what=f"decode {i}")
+
+
 def test_large_cursor_positions():
     """Positions far beyond the live length (holes only in position space)."""
     from harness import Pair
