@@ -276,6 +276,43 @@ def run_reference(args):
 # ----------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------
+def from_scratch_prefill(w, plan, mk, flush, args, seed_base):
+    """The refill workload's other arm: the text of round 0 (prefix + tail)
+    computed from an empty cache and zero states in one round, the dense
+    refill that the tail update avoids (§5.2).  Median device time of
+    max(3, steps / 8) runs after `warmup` untimed ones; before each run the
+    context is reset by a fork of an empty one and L2 is flushed, both
+    outside the timed events."""
+    import torch
+    s = w.shape
+    n_all = [a + b for a, b in zip(w.prefix_len, plan[0][3])]
+    tot = sum(n_all)
+    empty, fresh = mk(tot), mk(tot)
+    ins = W.device_round_inputs(w, seed_base + 7777, n_all)
+    outs = {l: torch.empty((tot, s.n_q_heads, s.head_dim) if k == W.ATTN else (tot, s.n_gdn_heads, s.d_v),
+                           dtype=torch.bfloat16, device="cuda") for l, k in enumerate(s.layer_kind)}
+    zero_cu = np.zeros(w.n_chars + 1, np.int32)
+    cu_all = np.concatenate([[0], np.cumsum(n_all)]).astype(np.int32)
+    stream = torch.cuda.current_stream()
+    evs = []
+    for i in range(args.warmup + max(3, args.steps // 8)):
+        fresh.fork_from(empty)
+        flush.fill_(i & 0x7F)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fresh.update_round(zero_cu, [], [], cu_all, ins, outs)
+        e1.record(stream)
+        if i >= args.warmup:
+            evs.append((e0, e1))
+    torch.cuda.synchronize()
+    fresh.check()
+    ms = float(np.median([a.elapsed_time(b) for a, b in evs]))
+    del ins, outs, empty, fresh
+    torch.cuda.empty_cache()
+    return {"what": "the same text as a from-scratch prefill: empty cache, zero states, one round",
+            "tokens": tot, "ms": ms, "runs": len(evs)}
+
+
 def run_kvm(args):
     import torch
     import torch.distributed as dist
@@ -408,6 +445,7 @@ def run_kvm(args):
     # per-kernel durations: the same steps again with per-launch events
     prof_ms, _, kernels, _, _, _ = timed(host_io=False, profile=True)
     e2e_ms, e2e_rids, _, _, _, e2e_steps = timed(host_io=True)
+    scratch = from_scratch_prefill(w, plan, mk, flush, args, seed_base) if args.workload == "refill" else None
     clocks.stop()
 
     toks_rank = sum(sum(rounds[r]["tails"]) for r in rids)
@@ -508,6 +546,10 @@ def run_kvm(args):
         "rooflines": rooflines,
         "clocks": clk,
     }
+    if scratch is not None:
+        scratch["tail_update_ms"] = total_ms / args.steps
+        scratch["ratio"] = scratch["ms"] / scratch["tail_update_ms"]
+        line["refill_from_scratch"] = scratch
     print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
