@@ -138,6 +138,42 @@ kvm_status kvm_spans_from_positions(kvm_ctx* ctx, int32_t b, int32_t n,
                                     const int64_t* pos_begin, const int64_t* pos_end,
                                     int32_t* span_begin, int32_t* span_end);
 
+/* ------------------------------------------------------------ host-only planning
+ * These touch no context and no device: they compute on the host what the
+ * hot-path calls plan before their first launch, so that a caller can check
+ * a round ahead of time and tests can check the planning on a machine
+ * without a GPU. */
+
+/* Eq. 2 on the host: validate one round's removal spans against the live
+ * lengths live host [n_chars] with exactly the checks of kvm_kv_compact
+ * (span_cu, span_begin, span_end as there), and report its effect: new_live
+ * host [n_chars] = L'_b = live_b minus the removed count, first_moved host
+ * [n_chars] = the first live index at or after which entries move (the first
+ * span's begin; L'_b when the character removes nothing).  Either output may
+ * be NULL.  Errors: KVM_E_INVAL, KVM_E_SPAN. */
+kvm_status kvm_plan_removal(int32_t n_chars, const int32_t* live, const int32_t* span_cu,
+                            const int32_t* span_begin, const int32_t* span_end, int32_t* new_live,
+                            int32_t* first_moved);
+
+/* The work partition kvm_tail_attn_prefill uses for one attention layer
+ * (Eq. 3), for live lengths L'_b live host [n_chars] (after removal) and
+ * tails tail_cu host [n_chars+1].  Query tiles hold 128 / g tail tokens of
+ * one KV head (g = n_q_heads / n_kv_heads) and are numbered (character, KV
+ * head, tile); tile t of character b attends to ceil((L'_b + last token of
+ * the tile + 1) / 64) 64-key tiles.  The (query tile, key tile) units, in
+ * that order, are cut into *n_blocks <= max_blocks contiguous ranges; block
+ * c processes units from (block_tile[c], block_key[c]) up to, not including,
+ * (block_tile[c+1], block_key[c+1]).  block_tile and block_key: host
+ * [max_blocks + 1].  *n_tiles = number of query tiles.  split_first_block
+ * host [max_blocks]: for each of the *n_split query tiles that several
+ * blocks share, the first block that starts inside it (its partials are
+ * merged by the combine kernel).  kvm_tail_attn_prefill uses max_blocks =
+ * min(320, the device's SM count).  Errors: KVM_E_INVAL, KVM_E_UNSUPPORTED. */
+kvm_status kvm_plan_attention(int32_t n_chars, const int32_t* live, const int32_t* tail_cu,
+                              int32_t n_q_heads, int32_t n_kv_heads, int32_t max_blocks,
+                              int32_t* n_blocks, int32_t* n_tiles, int32_t* block_tile,
+                              int32_t* block_key, int32_t* n_split, int32_t* split_first_block);
+
 /* ------------------------------------------------------------ hot path */
 
 /* Eq. 2: remove the live entries named by the spans from every attention

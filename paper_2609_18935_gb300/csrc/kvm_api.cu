@@ -191,24 +191,26 @@ struct SpanPlan {
     std::vector<int32_t> seg_start, seg_shift;
 };
 
-kvm_status plan_spans(const kvm_ctx* c, const int32_t* span_cu, const int32_t* sb, const int32_t* se,
-                      SpanPlan& pl) {
+// B characters with live lengths live[B] (host state, no device access).
+kvm_status plan_spans_for(int B, const int* live, const int32_t* span_cu, const int32_t* sb, const int32_t* se,
+                          SpanPlan& pl) {
     if (!span_cu) return fail(KVM_E_INVAL, "span_cu is NULL");
     if (span_cu[0] != 0) return fail(KVM_E_INVAL, "span_cu[0] must be 0");
-    const int total = span_cu[c->B];
+    const int total = span_cu[B];
     if (total < 0) return fail(KVM_E_INVAL, "negative span count");
     if (total > kMaxSpans) return fail(KVM_E_INVAL, "%d spans exceed the per-round limit %d", total, kMaxSpans);
     if (total > 0 && (!sb || !se)) return fail(KVM_E_INVAL, "span arrays are NULL");
-    pl.L_new.assign(c->B, 0);
-    pl.first.assign(c->B, 0);
-    pl.seg_off.assign(c->B, 0);
-    pl.n_seg.assign(c->B, 0);
+    pl.L_new.assign(B, 0);
+    pl.first.assign(B, 0);
+    pl.seg_off.assign(B, 0);
+    pl.n_seg.assign(B, 0);
     pl.seg_start.clear();
     pl.seg_shift.clear();
-    for (int b = 0; b < c->B; ++b) {
+    for (int b = 0; b < B; ++b) {
         const int s0 = span_cu[b], s1 = span_cu[b + 1];
-        if (s1 < s0) return fail(KVM_E_INVAL, "span_cu not monotone at character %d", b);
-        const int L = c->live[b];
+        if (s1 < s0 || s0 < 0 || s1 > total)
+            return fail(KVM_E_INVAL, "span_cu not monotone at character %d", b);
+        const int L = live[b];
         int removed = 0, prev_end = 0;
         pl.seg_off[b] = (int)pl.seg_start.size();
         pl.n_seg[b] = s1 - s0;
@@ -229,6 +231,92 @@ kvm_status plan_spans(const kvm_ctx* c, const int32_t* span_cu, const int32_t* s
         pl.first[b] = (s1 > s0) ? sb[s0] : pl.L_new[b];
     }
     return KVM_OK;
+}
+
+kvm_status plan_spans(const kvm_ctx* c, const int32_t* span_cu, const int32_t* sb, const int32_t* se,
+                      SpanPlan& pl) {
+    return plan_spans_for(c->B, c->live.data(), span_cu, sb, se, pl);
+}
+
+// The attention's work partition for one layer: query tiles numbered
+// (character, KV head, tile), each with the 64-key tiles it attends to
+// (every surviving entry plus the tail up to its last token).  Stream-K with
+// a cost model: block cc gets a contiguous range of (query tile, key tile)
+// units; a unit costs 1 and every segment a block starts (its first one, and
+// each query tile it enters) costs kSegmentCost more (Q staging, the
+// epilogue, the pipeline refill).  The ranges are cut greedily at a
+// per-block cost target, found by bisection so that exactly G blocks cover
+// the units with the least maximum cost.  Tiles shared by several blocks are
+// merged once, from the first block that starts inside them (split_cb).
+struct AttnPlan {
+    int n_tiles = 0, n_ctas = 0;
+    std::vector<int> n_qtiles, tile_off;             // per character
+    std::vector<int32_t> cta_tile, cta_k, split_cb;  // [n_ctas + 1], [n_ctas + 1], [number of split tiles]
+};
+
+void plan_attention(int B, const int* L_prev, const int* M, int Hkv, int tpt, int grid_cap, AttnPlan& pl) {
+    pl.n_qtiles.assign(B, 0);
+    pl.tile_off.assign(B, 0);
+    std::vector<int> nk_of;
+    int tiles = 0;
+    int64_t units = 0;
+    for (int b = 0; b < B; ++b) {
+        pl.n_qtiles[b] = (M[b] + tpt - 1) / tpt;
+        pl.tile_off[b] = tiles;
+        tiles += Hkv * pl.n_qtiles[b];
+    }
+    nk_of.reserve(tiles);
+    for (int b = 0; b < B; ++b)
+        for (int h = 0; h < Hkv; ++h)
+            for (int qt = 0; qt < pl.n_qtiles[b]; ++qt) {
+                nk_of.push_back((L_prev[b] + std::min(M[b], (qt + 1) * tpt) + 63) / 64);
+                units += nk_of.back();
+            }
+    pl.n_tiles = tiles;
+    const int G = (int)std::max<int64_t>(1, std::min<int64_t>(grid_cap, units / kMinUnitsPerCta));
+    pl.n_ctas = G;
+    pl.cta_tile.assign(G + 1, 0);
+    pl.cta_k.assign(G + 1, 0);
+    // blocks needed to cover everything with ranges of cost <= target; the
+    // cut points go to cta_tile / cta_k when `emit`
+    auto cover = [&](double target, bool emit) -> int {
+        int blocks = 1;
+        double cost = kSegmentCost;
+        for (int t = 0; t < (int)nk_of.size(); ++t) {
+            int k = 0;
+            if (t > 0) cost += kSegmentCost;                  // entering a new query tile
+            while (k < nk_of[t]) {
+                const double room = target - cost;
+                const int take = room >= nk_of[t] - k ? nk_of[t] - k : std::max(0, (int)room);
+                k += take;
+                cost += take;
+                if (k < nk_of[t] && (take == 0 || cost >= target)) {
+                    if (take == 0 && cost == kSegmentCost) {      // a block must take at least a unit
+                        ++k;
+                        cost += 1;
+                        if (k >= nk_of[t]) break;
+                    }
+                    if (emit && blocks <= G) { pl.cta_tile[blocks] = t; pl.cta_k[blocks] = k; }
+                    ++blocks;
+                    cost = kSegmentCost;
+                }
+            }
+        }
+        return blocks;
+    };
+    double lo = (double)units / G, hi = (double)units / G + 2.0 * kSegmentCost * (1 + tiles / G) + 1.0;
+    while (cover(hi, false) > G) hi *= 2;
+    for (int it = 0; it < 40 && hi - lo > 0.25; ++it) {
+        const double mid = 0.5 * (lo + hi);
+        if (cover(mid, false) <= G) hi = mid; else lo = mid;
+    }
+    const int used = cover(hi, true);
+    // fewer ranges than blocks: the spare blocks get empty ranges at the end
+    for (int cc = used; cc <= G; ++cc) { pl.cta_tile[cc] = tiles; pl.cta_k[cc] = 0; }
+    pl.split_cb.clear();
+    for (int cc = 1; cc < G; ++cc)
+        if (pl.cta_k[cc] > 0 && !(pl.cta_tile[cc - 1] == pl.cta_tile[cc] && pl.cta_k[cc - 1] > 0))
+            pl.split_cb.push_back(cc);
 }
 
 }  // namespace
@@ -486,6 +574,58 @@ extern "C" kvm_status kvm_get_live(kvm_ctx* c, int32_t b, int32_t* live, int64_t
     return KVM_OK;
 }
 
+// ============================================================================
+// host-only planning (no context, no device)
+// ============================================================================
+extern "C" kvm_status kvm_plan_removal(int32_t n_chars, const int32_t* live, const int32_t* span_cu,
+                                       const int32_t* span_begin, const int32_t* span_end, int32_t* new_live,
+                                       int32_t* first_moved) {
+    if (n_chars <= 0 || n_chars > kMaxChars) return fail(KVM_E_INVAL, "n_chars must be in [1,%d]", kMaxChars);
+    if (!live) return fail(KVM_E_INVAL, "live is NULL");
+    std::vector<int> L(live, live + n_chars);
+    for (int b = 0; b < n_chars; ++b)
+        if (L[b] < 0) return fail(KVM_E_INVAL, "negative live length at character %d", b);
+    SpanPlan pl;
+    const kvm_status st = plan_spans_for(n_chars, L.data(), span_cu, span_begin, span_end, pl);
+    if (st) return st;
+    for (int b = 0; b < n_chars; ++b) {
+        if (new_live) new_live[b] = pl.L_new[b];
+        if (first_moved) first_moved[b] = pl.first[b];
+    }
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_plan_attention(int32_t n_chars, const int32_t* live, const int32_t* tail_cu,
+                                         int32_t n_q_heads, int32_t n_kv_heads, int32_t max_blocks,
+                                         int32_t* n_blocks, int32_t* n_tiles, int32_t* block_tile,
+                                         int32_t* block_key, int32_t* n_split, int32_t* split_first_block) {
+    if (n_chars <= 0 || n_chars > kMaxChars) return fail(KVM_E_INVAL, "n_chars must be in [1,%d]", kMaxChars);
+    if (!live || !tail_cu || !n_blocks || !n_tiles || !block_tile || !block_key || !n_split || !split_first_block)
+        return fail(KVM_E_INVAL, "NULL argument");
+    if (n_kv_heads <= 0 || n_q_heads <= 0 || n_q_heads % n_kv_heads)
+        return fail(KVM_E_UNSUPPORTED, "n_q_heads must be a multiple of n_kv_heads");
+    const int g = n_q_heads / n_kv_heads;
+    if (g > 64 || (g & (g - 1))) return fail(KVM_E_UNSUPPORTED, "group size must be a power of two <= 64");
+    if (max_blocks <= 0 || max_blocks > kMaxAttnCtas)
+        return fail(KVM_E_INVAL, "max_blocks must be in [1,%d]", kMaxAttnCtas);
+    if (tail_cu[0] != 0) return fail(KVM_E_INVAL, "tail_cu[0] must be 0");
+    std::vector<int> L(live, live + n_chars), M(n_chars);
+    for (int b = 0; b < n_chars; ++b) {
+        M[b] = tail_cu[b + 1] - tail_cu[b];
+        if (M[b] < 0) return fail(KVM_E_INVAL, "tail_cu not monotone at character %d", b);
+        if (L[b] < 0) return fail(KVM_E_INVAL, "negative live length at character %d", b);
+    }
+    AttnPlan pl;
+    plan_attention(n_chars, L.data(), M.data(), n_kv_heads, kAttnRows / g, max_blocks, pl);
+    *n_blocks = pl.n_ctas;
+    *n_tiles = pl.n_tiles;
+    std::copy(pl.cta_tile.begin(), pl.cta_tile.end(), block_tile);
+    std::copy(pl.cta_k.begin(), pl.cta_k.end(), block_key);
+    *n_split = (int32_t)pl.split_cb.size();
+    std::copy(pl.split_cb.begin(), pl.split_cb.end(), split_first_block);
+    return KVM_OK;
+}
+
 extern "C" kvm_status kvm_spans_from_positions(kvm_ctx* c, int32_t b, int32_t n, const int64_t* pb,
                                                const int64_t* pe, int32_t* sb, int32_t* se) {
     if (!c) return fail(KVM_E_INVAL, "NULL context");
@@ -663,86 +803,27 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
     p.err = c->err;
     p.diag = c->diag;
     for (int d = 0; d < c->R / 2; ++d) p.inv_freq[d] = c->inv_freq[d];
-    // query tiles (character, KV head, tile) and their 64-key tiles
-    const int tpt = p.tok_per_tile;
-    int tiles = 0;
-    int64_t units = 0;
+    std::vector<int> Ms(c->B);
     for (int b = 0; b < c->B; ++b) {
         AttnChar& ch = p.ch[b];
         ch.L_prev = c->live[b];
-        ch.M = tail_cu[b + 1] - tail_cu[b];
+        ch.M = Ms[b] = tail_cu[b + 1] - tail_cu[b];
         ch.tail_off = tail_cu[b];
         ch.cap_off = c->cap_off[b];
         ch.p = c->cursor[b];
-        ch.n_qtiles = (ch.M + tpt - 1) / tpt;
-        ch.tile_off = tiles;
-        tiles += c->Hkv * ch.n_qtiles;
-        for (int qt = 0; qt < ch.n_qtiles; ++qt)
-            units += (int64_t)c->Hkv * ((ch.L_prev + std::min(ch.M, (qt + 1) * tpt) + 63) / 64);
     }
-    p.n_tiles = tiles;
-    // stream-K with a cost model: block cc gets a contiguous range of
-    // (query tile, key tile) units; a unit costs 1 and every segment a block
-    // starts (its first one, and each query tile it enters) costs
-    // kSegmentCost more (Q staging, the epilogue, the pipeline refill).  The
-    // ranges are cut greedily at a per-block cost target, found by bisection
-    // so that exactly G blocks cover the units with the least maximum cost.
-    const int G = (int)std::max<int64_t>(1, std::min<int64_t>(attention_grid_cap(c->num_sms, c->D),
-                                                              units / kMinUnitsPerCta));
-    p.n_ctas = G;
-    {
-        std::vector<int> nk_of;
-        nk_of.reserve(tiles);
-        for (int b = 0; b < c->B; ++b) {
-            const AttnChar& ch = p.ch[b];
-            for (int h = 0; h < c->Hkv; ++h)
-                for (int qt = 0; qt < ch.n_qtiles; ++qt)
-                    nk_of.push_back((ch.L_prev + std::min(ch.M, (qt + 1) * tpt) + 63) / 64);
-        }
-        // blocks needed to cover everything with ranges of cost <= target; the
-        // cut points go to p.cta_tile / p.cta_k when `emit`
-        auto cover = [&](double target, bool emit) -> int {
-            int blocks = 1;
-            double cost = kSegmentCost;
-            if (emit) { p.cta_tile[0] = 0; p.cta_k[0] = 0; }
-            for (int t = 0; t < (int)nk_of.size(); ++t) {
-                int k = 0;
-                if (t > 0) cost += kSegmentCost;                  // entering a new query tile
-                while (k < nk_of[t]) {
-                    const double room = target - cost;
-                    const int take = room >= nk_of[t] - k ? nk_of[t] - k : std::max(0, (int)room);
-                    k += take;
-                    cost += take;
-                    if (k < nk_of[t] && (take == 0 || cost >= target)) {
-                        if (take == 0 && cost == kSegmentCost) {      // a block must take at least a unit
-                            ++k;
-                            cost += 1;
-                            if (k >= nk_of[t]) break;
-                        }
-                        if (emit && blocks <= G) { p.cta_tile[blocks] = t; p.cta_k[blocks] = k; }
-                        ++blocks;
-                        cost = kSegmentCost;
-                    }
-                }
-            }
-            return blocks;
-        };
-        double lo = (double)units / G, hi = (double)units / G + 2.0 * kSegmentCost * (1 + tiles / G) + 1.0;
-        while (cover(hi, false) > G) hi *= 2;
-        for (int it = 0; it < 40 && hi - lo > 0.25; ++it) {
-            const double mid = 0.5 * (lo + hi);
-            if (cover(mid, false) <= G) hi = mid; else lo = mid;
-        }
-        const int used = cover(hi, true);
-        // fewer ranges than blocks: the spare blocks get empty ranges at the end
-        for (int cc = used; cc <= G; ++cc) { p.cta_tile[cc] = tiles; p.cta_k[cc] = 0; }
+    AttnPlan pl;
+    plan_attention(c->B, c->live.data(), Ms.data(), c->Hkv, p.tok_per_tile, attention_grid_cap(c->num_sms, c->D), pl);
+    for (int b = 0; b < c->B; ++b) {
+        p.ch[b].n_qtiles = pl.n_qtiles[b];
+        p.ch[b].tile_off = pl.tile_off[b];
     }
-    // tiles shared by several blocks: each is merged once, from the first
-    // block that starts inside it
-    p.n_split_tiles = 0;
-    for (int cc = 1; cc < G; ++cc)
-        if (p.cta_k[cc] > 0 && !(p.cta_tile[cc - 1] == p.cta_tile[cc] && p.cta_k[cc - 1] > 0))
-            p.split_cb[p.n_split_tiles++] = cc;
+    p.n_tiles = pl.n_tiles;
+    p.n_ctas = pl.n_ctas;
+    std::copy(pl.cta_tile.begin(), pl.cta_tile.end(), p.cta_tile);
+    std::copy(pl.cta_k.begin(), pl.cta_k.end(), p.cta_k);
+    p.n_split_tiles = (int)pl.split_cb.size();
+    std::copy(pl.split_cb.begin(), pl.split_cb.end(), p.split_cb);
     const bool split_tiles = p.n_split_tiles > 0;
 
     int ps = prof_begin(c, KVM_K_ROPE_APPEND, s);

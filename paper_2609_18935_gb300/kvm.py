@@ -74,6 +74,11 @@ _SIGS = {
     "kvm_check": (C.c_int, [C.c_void_p, C.c_void_p]),
     "kvm_launch_count": (C.c_int64, [C.c_void_p]),
     "kvm_fork": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "kvm_plan_removal": (C.c_int, [C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32),
+                                   C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
+    "kvm_plan_attention": (C.c_int, [C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.c_int32, C.c_int32,
+                                     C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32),
+                                     C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
     "kvm_kv_compact_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int64, C.c_int32,
                                          C.c_int32, C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32),
                                          C.POINTER(C.c_int32), C.c_void_p]),
@@ -153,6 +158,32 @@ def kv_compact_noalloc(K, V, positions, live, span_begin, span_end, stream=None)
                                        _dptr(positions, torch.int32), n_slabs, rows, D, int(live), len(sb),
                                        _p32(sb), _p32(se), C.byref(new_live), _stream(stream)))
     return new_live.value
+
+
+def plan_removal(live, span_cu, span_begin, span_end):
+    """kvm_plan_removal: (new live lengths, first moved index) per character;
+    raises KvmError with the library's status on invalid spans."""
+    load_library()
+    L = _i32(live)
+    cu, sb, se = _i32(span_cu), _i32(span_begin), _i32(span_end)
+    new_live, first = np.zeros(len(L), np.int32), np.zeros(len(L), np.int32)
+    _check(_lib.kvm_plan_removal(len(L), _p32(L), _p32(cu), _p32(sb) if len(sb) else None,
+                                 _p32(se) if len(se) else None, _p32(new_live), _p32(first)))
+    return new_live, first
+
+
+def plan_attention(live, tail_cu, n_q_heads, n_kv_heads, max_blocks):
+    """kvm_plan_attention: the attention's work partition for one layer."""
+    load_library()
+    L, cu = _i32(live), _i32(tail_cu)
+    tile, key = np.zeros(max_blocks + 1, np.int32), np.zeros(max_blocks + 1, np.int32)
+    split = np.zeros(max_blocks, np.int32)
+    nb, nt, ns = C.c_int32(), C.c_int32(), C.c_int32()
+    _check(_lib.kvm_plan_attention(len(L), _p32(L), _p32(cu), int(n_q_heads), int(n_kv_heads), int(max_blocks),
+                                   C.byref(nb), C.byref(nt), _p32(tile), _p32(key), C.byref(ns), _p32(split)))
+    n = nb.value
+    return {"n_blocks": n, "n_tiles": nt.value, "block_tile": tile[:n + 1].copy(), "block_key": key[:n + 1].copy(),
+            "split_first_block": split[:ns.value].copy()}
 
 
 def pinned_layer_inputs(inputs):
