@@ -38,6 +38,7 @@ from workload import synth as W  # noqa: E402
 
 METRIC = "tail tokens/sec per maintenance round and ms/round; % of HBM/tensor roofline"
 UNIT = "tail tokens/s"
+PROFILE_STEPS = 256   # steps of the per-kernel pass: ~10 launches each, within the library's 4096-event pool
 
 WORKLOAD_TEXT = {
     "tiny": "1 delta-rule (8 heads, d 64) + 1 GQA attention layer (8/2 heads, D 64, RoPE 64), prefix 512, "
@@ -280,7 +281,7 @@ def from_scratch_prefill(w, plan, mk, flush, args, seed_base):
     """The refill workload's other arm: the text of round 0 (prefix + tail)
     computed from an empty cache and zero states in one round, the dense
     refill that the tail update avoids (§5.2).  Median device time of
-    max(3, steps / 8) runs after `warmup` untimed ones; before each run the
+    max(3, min(16, steps / 8)) runs after `warmup` untimed ones; before each run the
     context is reset by a fork of an empty one and L2 is flushed, both
     outside the timed events."""
     import torch
@@ -295,7 +296,7 @@ def from_scratch_prefill(w, plan, mk, flush, args, seed_base):
     cu_all = np.concatenate([[0], np.cumsum(n_all)]).astype(np.int32)
     stream = torch.cuda.current_stream()
     evs = []
-    for i in range(args.warmup + max(3, args.steps // 8)):
+    for i in range(args.warmup + max(3, min(16, args.steps // 8))):
         fresh.fork_from(empty)
         flush.fill_(i & 0x7F)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -407,7 +408,10 @@ def run_kvm(args):
         """Warm-up steps, then K timed steps.  With `profile`, every library
         launch is bracketed by CUDA events (per-kernel durations); those
         events sit between kernels and keep consecutive launches from
-        overlapping, so the headline steps run without them."""
+        overlapping, so the headline steps run without them.  The profiled
+        pass runs at most PROFILE_STEPS steps, so that its launches stay
+        within the library's event pool."""
+        n_steps = min(args.steps, PROFILE_STEPS) if profile else args.steps
         for i in range(args.warmup):
             one_step(i, host_io)
         work.check()
@@ -419,7 +423,7 @@ def run_kvm(args):
         work.profile_enable(profile)
         work.profile_read(0, reset=True)
         t0 = time.time()
-        evs = [one_step(i, host_io) for i in range(args.steps)]
+        evs = [one_step(i, host_io) for i in range(n_steps)]
         torch.cuda.synchronize()
         t1 = time.time()
         if world > 1:
@@ -442,8 +446,8 @@ def run_kvm(args):
     time.sleep(0.3)
     total_ms, rids, _, launches, (t0, t1), _ = timed(host_io=False)
     clk = clocks.summary(t0, t1)
-    # per-kernel durations: the same steps again with per-launch events
-    prof_ms, _, kernels, _, _, _ = timed(host_io=False, profile=True)
+    # per-kernel durations: the same steps again (at most PROFILE_STEPS) with per-launch events
+    prof_ms, prof_rids, kernels, _, _, _ = timed(host_io=False, profile=True)
     e2e_ms, e2e_rids, _, _, _, e2e_steps = timed(host_io=True)
     scratch = from_scratch_prefill(w, plan, mk, flush, args, seed_base) if args.workload == "refill" else None
     clocks.stop()
@@ -453,12 +457,12 @@ def run_kvm(args):
     e2e_value = job_throughput(world, sum(sum(rounds[r]["tails"]) for r in e2e_rids), e2e_ms)
     hbm, tc_burst, tc_sust, peak_src = load_peaks()
     n_attn, n_gdn = len(s.attn_layers), len(s.gdn_layers)
-    # algorithmic work of every kernel family over the timed steps
+    # algorithmic work of every kernel family over the steps of the per-kernel pass
     work = {
-        "tail_attention": ("tensor", sum(rounds[r]["attn_flops"] * n_attn for r in rids)),
-        "gdn": ("hbm", sum(rounds[r]["gdn_bytes"] * n_gdn for r in rids)),
-        "kv_compact": ("hbm", sum(rounds[r]["compact_bytes"] for r in rids)),
-        "rope_append": ("hbm", sum(rounds[r]["rope_bytes"] * n_attn for r in rids)),
+        "tail_attention": ("tensor", sum(rounds[r]["attn_flops"] * n_attn for r in prof_rids)),
+        "gdn": ("hbm", sum(rounds[r]["gdn_bytes"] * n_gdn for r in prof_rids)),
+        "kv_compact": ("hbm", sum(rounds[r]["compact_bytes"] for r in prof_rids)),
+        "rope_append": ("hbm", sum(rounds[r]["rope_bytes"] * n_attn for r in prof_rids)),
     }
     fam = {k: dict(v) for k, v in kernels.items()}
     if "gdn_chunk_scan" in fam:
@@ -542,7 +546,7 @@ def run_kvm(args):
         "kernels": per_kernel,
         "kernel_timing": ("per-launch CUDA events in a second pass over the same steps (events between "
                           "kernels stop launches from overlapping, so the headline pass runs without them); "
-                          f"that pass took {prof_ms / args.steps:.4f} ms per step"),
+                          f"that pass took {prof_ms / len(prof_rids):.4f} ms per step over {len(prof_rids)} steps"),
         "rooflines": rooflines,
         "clocks": clk,
     }

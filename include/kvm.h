@@ -304,10 +304,11 @@ kvm_status kvm_fork(kvm_ctx* dst, const kvm_ctx* src, void* stream);
 /* Per-kernel timing for diagnostics.  While enabled, each kernel launch of
  * the library is bracketed by a pair of CUDA events on its stream.
  * kvm_profile_read synchronizes the device and returns, for one kernel
- * family (KVM_K_*), the number of launches and their summed device time in
- * milliseconds since the last reset; reset != 0 clears every family.
+ * family (KVM_K_*), the number of timed launches and their summed device
+ * time in milliseconds since the last reset; reset != 0 clears every family.
  * Events come from a pool made at enable time (4096 launches between
- * reads); launches beyond it are counted but not timed. */
+ * reads); launches beyond it are neither timed nor counted here
+ * (kvm_launch_count counts every launch). */
 enum { KVM_K_COMPACT = 0, KVM_K_ROPE_APPEND = 1, KVM_K_ATTENTION = 2, KVM_K_ATTN_COMBINE = 3,
        KVM_K_GDN = 4, KVM_K_GATHER = 5, KVM_K_GDN_PREP = 6, KVM_K_COUNT = 7 };
 kvm_status kvm_profile_enable(kvm_ctx* ctx, int32_t enable);

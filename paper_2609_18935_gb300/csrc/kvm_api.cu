@@ -116,7 +116,6 @@ struct kvm_ctx {
     bool prof = false;
     std::vector<cudaEvent_t> ev;          // 2 per timed launch
     std::vector<int> ev_kind;             // kind of each recorded pair
-    int64_t prof_launches[KVM_K_COUNT] = {};
 };
 
 namespace {
@@ -173,7 +172,6 @@ constexpr int kProfPool = 4096;
 int prof_begin(kvm_ctx* c, int kind, cudaStream_t s) {
     ++c->launches;
     if (!c->prof) return -1;
-    ++c->prof_launches[kind];
     const int slot = (int)c->ev_kind.size();
     if (slot >= kProfPool) return -1;
     c->ev_kind.push_back(kind);
@@ -1153,18 +1151,17 @@ extern "C" kvm_status kvm_profile_read(kvm_ctx* c, int32_t kernel, int64_t* laun
     if (kernel < 0 || kernel >= KVM_K_COUNT) return fail(KVM_E_INVAL, "kernel family %d out of range", kernel);
     CUDA_TRY(cudaDeviceSynchronize());
     double ms = 0.0;
+    int64_t timed = 0;                     // launches that got a pair of events
     for (size_t i = 0; i < c->ev_kind.size(); ++i) {
         if (c->ev_kind[i] != kernel) continue;
         float t = 0.f;
         CUDA_TRY(cudaEventElapsedTime(&t, c->ev[2 * i], c->ev[2 * i + 1]));
         ms += t;
+        ++timed;
     }
-    if (launches) *launches = c->prof_launches[kernel];
+    if (launches) *launches = timed;
     if (total_ms) *total_ms = ms;
-    if (reset) {
-        c->ev_kind.clear();
-        for (auto& n : c->prof_launches) n = 0;
-    }
+    if (reset) c->ev_kind.clear();
     return KVM_OK;
 }
 
