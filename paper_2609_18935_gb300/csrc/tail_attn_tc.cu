@@ -530,7 +530,7 @@ void launch_tail_attention(const AttnParams& p, cudaStream_t s) {
     }
 }
 
-// One block per SM: 320 threads of about 128 registers leave no room for a
+// One block per SM: 384 threads of about 150 registers leave no room for a
 // second (and head_dim 256 needs all of TMEM and shared memory).
 int attention_ctas_per_sm(int) { return 1; }
 
