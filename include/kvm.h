@@ -155,6 +155,13 @@ kvm_status kvm_plan_removal(int32_t n_chars, const int32_t* live, const int32_t*
                             const int32_t* span_begin, const int32_t* span_end, int32_t* new_live,
                             int32_t* first_moved);
 
+/* kvm_spans_from_positions on a caller's copy of one character's live
+ * positions: positions host [live], strictly increasing.  Same mapping,
+ * checks and errors (KVM_E_INVAL for bad arguments, KVM_E_SPAN for ranges). */
+kvm_status kvm_plan_spans_from_positions(int32_t live, const int32_t* positions, int32_t n,
+                                         const int64_t* pos_begin, const int64_t* pos_end,
+                                         int32_t* span_begin, int32_t* span_end);
+
 /* The work partition kvm_tail_attn_prefill uses for one attention layer
  * (Eq. 3), for live lengths L'_b live host [n_chars] (after removal) and
  * tails tail_cu host [n_chars+1].  Query tiles hold 128 / g tail tokens of

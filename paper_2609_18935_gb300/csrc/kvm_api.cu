@@ -624,25 +624,43 @@ extern "C" kvm_status kvm_plan_attention(int32_t n_chars, const int32_t* live, c
     return KVM_OK;
 }
 
-extern "C" kvm_status kvm_spans_from_positions(kvm_ctx* c, int32_t b, int32_t n, const int64_t* pb,
-                                               const int64_t* pe, int32_t* sb, int32_t* se) {
-    if (!c) return fail(KVM_E_INVAL, "NULL context");
-    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+namespace {
+// Position ranges -> live-index spans over the sorted live positions P[live].
+kvm_status spans_from_positions(const int32_t* P, int live, int32_t n, const int64_t* pb, const int64_t* pe,
+                                int32_t* sb, int32_t* se) {
     if (n < 0) return fail(KVM_E_INVAL, "negative count");
     if (n > 0 && (!pb || !pe || !sb || !se)) return fail(KVM_E_INVAL, "NULL argument");
-    const std::vector<int32_t>& P = c->hpos[b];
     int64_t prev_end = INT64_MIN;
     for (int i = 0; i < n; ++i) {
         if (pb[i] >= pe[i]) return fail(KVM_E_SPAN, "position range %d is empty", i);
         if (pb[i] < prev_end) return fail(KVM_E_SPAN, "position range %d overlaps or precedes the previous one", i);
         prev_end = pe[i];
-        const int lo = (int)(std::lower_bound(P.begin(), P.end(), pb[i]) - P.begin());
-        const int hi = (int)(std::lower_bound(P.begin(), P.end(), pe[i]) - P.begin());
+        const int lo = (int)(std::lower_bound(P, P + live, pb[i]) - P);
+        const int hi = (int)(std::lower_bound(P, P + live, pe[i]) - P);
         if (hi <= lo) return fail(KVM_E_SPAN, "position range %d covers no live entry", i);
         sb[i] = lo;
         se[i] = hi;
     }
     return KVM_OK;
+}
+}  // namespace
+
+extern "C" kvm_status kvm_spans_from_positions(kvm_ctx* c, int32_t b, int32_t n, const int64_t* pb,
+                                               const int64_t* pe, int32_t* sb, int32_t* se) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    const std::vector<int32_t>& P = c->hpos[b];
+    return spans_from_positions(P.data(), (int)P.size(), n, pb, pe, sb, se);
+}
+
+extern "C" kvm_status kvm_plan_spans_from_positions(int32_t live, const int32_t* positions, int32_t n,
+                                                    const int64_t* pos_begin, const int64_t* pos_end,
+                                                    int32_t* span_begin, int32_t* span_end) {
+    if (live < 0) return fail(KVM_E_INVAL, "negative live length");
+    if (live > 0 && !positions) return fail(KVM_E_INVAL, "positions is NULL");
+    for (int i = 1; i < live; ++i)
+        if (positions[i] <= positions[i - 1]) return fail(KVM_E_INVAL, "positions must be strictly increasing");
+    return spans_from_positions(positions, live, n, pos_begin, pos_end, span_begin, span_end);
 }
 
 // ============================================================================

@@ -76,6 +76,8 @@ _SIGS = {
     "kvm_fork": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "kvm_plan_removal": (C.c_int, [C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32),
                                    C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
+    "kvm_plan_spans_from_positions": (C.c_int, [C.c_int32, C.POINTER(C.c_int32), C.c_int32, C.POINTER(C.c_int64),
+                                                C.POINTER(C.c_int64), C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
     "kvm_plan_attention": (C.c_int, [C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.c_int32, C.c_int32,
                                      C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32),
                                      C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
@@ -170,6 +172,20 @@ def plan_removal(live, span_cu, span_begin, span_end):
     _check(_lib.kvm_plan_removal(len(L), _p32(L), _p32(cu), _p32(sb) if len(sb) else None,
                                  _p32(se) if len(se) else None, _p32(new_live), _p32(first)))
     return new_live, first
+
+
+def plan_spans_from_positions(positions, pos_begin, pos_end):
+    """kvm_plan_spans_from_positions: live-index spans (begin, end) of the
+    position ranges [pos_begin, pos_end) over one character's live positions."""
+    load_library()
+    P = _i32(positions)
+    pb = np.ascontiguousarray(np.asarray(pos_begin, dtype=np.int64))
+    pe = np.ascontiguousarray(np.asarray(pos_end, dtype=np.int64))
+    sb, se = np.zeros(len(pb), np.int32), np.zeros(len(pb), np.int32)
+    p64 = lambda a: a.ctypes.data_as(C.POINTER(C.c_int64))
+    _check(_lib.kvm_plan_spans_from_positions(len(P), _p32(P) if len(P) else None, len(pb), p64(pb), p64(pe),
+                                              _p32(sb), _p32(se)))
+    return sb, se
 
 
 def plan_attention(live, tail_cu, n_q_heads, n_kv_heads, max_blocks):

@@ -191,3 +191,45 @@ def test_plan_attention_rejects_bad_shapes():
         with pytest.raises(kvm.KvmError) as ei:
             kvm.plan_attention(*args)
         assert ei.value.code == code, args
+
+
+def test_spans_from_positions_match_brute_force():
+    """Position ranges [b, e) map to the live indices whose positions lie in
+    them (the paper checks deletion ranges against live spans, §4.2): holes
+    in the positions are skipped, and a range must be non-empty, in order,
+    and cover at least one live entry."""
+    rng = np.random.default_rng(479547)
+    for trial in range(300):
+        live = int(rng.integers(0, 60))
+        positions = np.sort(rng.choice(np.arange(400), size=live, replace=False)).astype(np.int32)
+        n = int(rng.integers(1, 5))
+        cuts = np.sort(rng.integers(-5, 410, size=2 * n))
+        pb, pe = cuts[0::2].tolist(), cuts[1::2].tolist()
+        if trial % 5 == 0 and n >= 2:                        # out of order
+            pb[0], pb[1], pe[0], pe[1] = pb[1], pb[0], pe[1], pe[0]
+        expect, prev_end, bad = [], None, False
+        for b, e in zip(pb, pe):
+            idx = np.flatnonzero((positions >= b) & (positions < e))
+            if b >= e or (prev_end is not None and b < prev_end) or idx.size == 0:
+                bad = True
+                break
+            prev_end = e
+            expect.append((int(idx[0]), int(idx[-1]) + 1))
+        if bad:
+            with pytest.raises(kvm.KvmError) as ei:
+                kvm.plan_spans_from_positions(positions, pb, pe)
+            assert ei.value.code == KVM_E_SPAN, (trial, positions, pb, pe)
+            continue
+        sb, se = kvm.plan_spans_from_positions(positions, pb, pe)
+        assert list(zip(sb.tolist(), se.tolist())) == expect
+        keep = O.keep_mask(live, sb, se)                     # the spans are a valid removal
+        in_ranges = np.zeros(live, bool)
+        for b, e in zip(pb, pe):
+            in_ranges |= (positions >= b) & (positions < e)
+        assert np.array_equal(~keep, in_ranges)
+
+
+def test_spans_from_positions_rejects_bad_positions():
+    with pytest.raises(kvm.KvmError) as ei:
+        kvm.plan_spans_from_positions([3, 3, 4], [0], [5])    # not strictly increasing
+    assert ei.value.code == KVM_E_INVAL
