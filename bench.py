@@ -5,13 +5,15 @@ A step is one maintenance round (every hot-path row): removal of superseded KV
 by compaction in every attention layer, then every layer in model order
 (RoPE at the true tail + cache append + causal GQA attention for attention
 layers; chunked gated delta rule from the carried state for recurrent
-layers), then the cursor advance.  Default workload ("npc"): 4 layers in a
-3:1 delta:attention pattern (delta 16 heads, d_k = d_v = 128; attention 16
-query / 2 KV heads, head_dim 256, RoPE on 64 dims), prefix 8192 built by a
-GPU refill, 8 chained rounds each removing 1-4 spans totalling ~5% and
-appending 256 tail tokens.  Steps cycle through the chain; before round 0 of
-each chain the working state is forked from the prefix root and before every
-step L2 is flushed (a 256 MiB write), both outside the timed events.
+layers), then the cursor advance.  Default workload ("long", the largest
+single-GPU configuration): 48 layers in a 3:1 delta:attention pattern (delta
+16 heads, d_k = d_v = 128; attention 16 query / 2 KV heads, head_dim 256,
+RoPE on 64 dims), a 32768-token prefix built by a GPU refill, one round
+removing 3% of the entries in 10 spans and appending 1024 tail tokens.
+`--workload npc|pop|refill|tiny` selects the other configurations.  Steps
+cycle through the workload's chain of rounds; before round 0 of each chain
+the working state is forked from the prefix root and before every step L2 is
+flushed (a 256 MiB write), both outside the timed events.
 
 Prints one JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle
 on a bounded sample of the same workload instead.
@@ -36,9 +38,14 @@ if ROOT not in sys.path:
 
 from workload import synth as W  # noqa: E402
 
+# tail tokens per step of the reference arm and of the cpu_baseline sample
+# (one hybrid block of character 0's round 0): a reference step takes a few
+# seconds, the cpu_baseline sample 10-30 s on 16 cores
+REFERENCE_TOKENS = {"tiny": 16, "npc": 8, "long": 4, "pop": 8, "refill": 8}
+CPU_BASELINE_TOKENS = {"tiny": 64, "npc": 96, "long": 48, "pop": 96, "refill": 64}
 METRIC = "tail tokens/sec per maintenance round and ms/round; % of HBM/tensor roofline"
 UNIT = "tail tokens/s"
-PROFILE_STEPS = 256   # steps of the per-kernel pass: ~10 launches each, within the library's 4096-event pool
+EVENT_POOL = 4096     # launches the library can time between two reads (kvm_profile_read)
 
 WORKLOAD_TEXT = {
     "tiny": "1 delta-rule (8 heads, d 64) + 1 GQA attention layer (8/2 heads, D 64, RoPE 64), prefix 512, "
@@ -180,30 +187,62 @@ class ClockSampler:
 # ----------------------------------------------------------------------------
 # CPU oracle sample (cpu_baseline leg and the reference arm)
 # ----------------------------------------------------------------------------
-def oracle_sample(w, m_sample: int):
-    """Time the fp64 oracle on round 0 of character 0, restricted to the first
-    m_sample tail tokens: compaction of every attention layer + every layer.
-    Returns (seconds, tail tokens)."""
+def oracle_block(w):
+    """Layers of the CPU sample: the first hybrid block of the stack (three
+    delta-rule layers and one attention layer in the 3:1 pattern; the whole
+    stack when it is shorter), and how many such blocks the stack has."""
+    kinds = w.shape.layer_kind
+    n = min(4, len(kinds))
+    return list(range(n)), len(kinds) / n
+
+
+def oracle_state(w):
+    """The fp64 oracle's state of character 0 before round 0, restricted to
+    the sample's layers (prefix cache and recurrent states as the GPU arm
+    draws them)."""
     from oracle import kvm_oracle as O
     s = w.shape
     N = w.prefix_len[0]
+    layers, _ = oracle_block(w)
     caches, states = {}, {}
-    for l in s.attn_layers:
-        K, V, pos = W.prefix_cache(w, 0, l, N)
-        caches[l] = O.AttnCache(O.bf16_to_f64(K), O.bf16_to_f64(V), pos)
-    for l in s.gdn_layers:
-        states[l] = O.f32_to_f64(W.prefix_state(w, 0, l))
-    st = O.CharacterState(caches, states, N)
+    for l in layers:
+        if s.layer_kind[l] == W.ATTN:
+            K, V, pos = W.prefix_cache(w, 0, l, N)
+            caches[l] = O.AttnCache(O.bf16_to_f64(K), O.bf16_to_f64(V), pos)
+        else:
+            states[l] = O.f32_to_f64(W.prefix_state(w, 0, l))
+    return O.CharacterState(caches, states, N)
+
+
+def oracle_sample(w, st, m_sample: int):
+    """Time the fp64 oracle on round 0 of character 0 for the sample's layers
+    (oracle_block), restricted to the first m_sample tail tokens: compaction
+    of the block's attention layer, then every layer of the block.  Returns
+    (seconds, tail tokens, blocks in the stack): the whole stack takes about
+    `blocks` times as long, since its blocks have the same shapes."""
+    from oracle import kvm_oracle as O
+    s = w.shape
+    N = w.prefix_len[0]
+    layers, blocks = oracle_block(w)
     cu, sb, se, tails = W.round_plan(w, 0, [N] + [0] * (w.n_chars - 1))
     m = min(m_sample, tails[0])
-    full = W.tail_inputs(w, 0, [m])
+    full = W.tail_inputs(w, 0, [m], layers=layers)
     ins = {}
-    for l, kind in enumerate(s.layer_kind):
-        x = full[l]
-        ins[l] = {k: (O.bf16_to_f64(v) if v.dtype == np.uint16 else O.f32_to_f64(v)) for k, v in x.items()}
+    for l in layers:
+        ins[l] = {k: (O.bf16_to_f64(v) if v.dtype == np.uint16 else O.f32_to_f64(v)) for k, v in full[l].items()}
+    kinds = [s.layer_kind[l] for l in layers]
     t0 = time.perf_counter()
-    O.maintenance_round(st, s.layer_kind, sb[cu[0]:cu[1]], se[cu[0]:cu[1]], ins, s.rotary_dim, s.rope_theta)
-    return time.perf_counter() - t0, m
+    O.maintenance_round(st, kinds, sb[cu[0]:cu[1]], se[cu[0]:cu[1]], ins, s.rotary_dim, s.rope_theta)
+    return time.perf_counter() - t0, m, blocks
+
+
+def sample_text(w, m, secs=None):
+    layers, blocks = oracle_block(w)
+    txt = (f"character 0, round 0 of the workload (prefix {w.prefix_len[0]}): compaction + layers "
+           f"{layers[0]}-{layers[-1]} (one 3:1 hybrid block) for the first {m} tail tokens, fp64 numpy; "
+           f"tokens/s scaled to the {len(w.shape.layer_kind)}-layer stack by its {blocks:g} blocks of the "
+           f"same shapes")
+    return txt + (f"; {secs:.1f} s" if secs is not None else "")
 
 
 def blas_threads() -> int:
@@ -248,28 +287,35 @@ def job_throughput(world: int, tokens_per_rank: float, ms: float) -> float:
     return world * tokens_per_rank / (ms / 1e3)
 
 
+def workload_config(w, args, world):
+    s = w.shape
+    return {"workload": WORKLOAD_TEXT[args.workload], "name": args.workload, "chars": w.n_chars,
+            "layers": len(s.layer_kind), "chain_rounds": w.rounds,
+            "l2": "flushed before every step (256 MiB write), outside the timed events",
+            "parallelism": f"{world} independent replica(s), characters per rank fixed"}
+
+
 def run_reference(args):
-    rank, _, _ = dist_env()
+    rank, world, _ = dist_env()
     if rank != 0:
         return
     w = W.make_workload(args.workload)
-    m = 8
+    m = REFERENCE_TOKENS[args.workload]
+    st = oracle_state(w)
     for _ in range(args.warmup):
-        oracle_sample(w, m)
+        oracle_sample(w, st, m)
     secs, toks = 0.0, 0
     for _ in range(args.steps):
-        t, n = oracle_sample(w, m)
-        secs += t
+        t, n, blocks = oracle_sample(w, st, m)
+        secs += t * blocks
         toks += n
     value = toks / secs
-    sample = (f"character 0, round 0 of the workload: compaction + all {len(w.shape.layer_kind)} layers for "
-              f"the first {m} tail tokens (prefix {w.prefix_len[0]}), fp64 numpy")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": WORKLOAD_TEXT[args.workload]},
+            "data": "synthetic", "config": workload_config(w, args, world),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
-                             "sample": sample},
+                             "sample": "each step: " + sample_text(w, m)},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -409,9 +455,9 @@ def run_kvm(args):
         launch is bracketed by CUDA events (per-kernel durations); those
         events sit between kernels and keep consecutive launches from
         overlapping, so the headline steps run without them.  The profiled
-        pass runs at most PROFILE_STEPS steps, so that its launches stay
-        within the library's event pool."""
-        n_steps = min(args.steps, PROFILE_STEPS) if profile else args.steps
+        pass runs as many steps as the library's event pool can time (all
+        of them when they fit)."""
+        n_steps = min(args.steps, max(1, EVENT_POOL // max(1, launches_per_step))) if profile else args.steps
         for i in range(args.warmup):
             one_step(i, host_io)
         work.check()
@@ -444,9 +490,11 @@ def run_kvm(args):
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
+    launches_per_step = 1
     total_ms, rids, _, launches, (t0, t1), _ = timed(host_io=False)
+    launches_per_step = -(-launches // args.steps)
     clk = clocks.summary(t0, t1)
-    # per-kernel durations: the same steps again (at most PROFILE_STEPS) with per-launch events
+    # per-kernel durations: the same steps again (as many as the event pool times) with per-launch events
     prof_ms, prof_rids, kernels, _, _, _ = timed(host_io=False, profile=True)
     e2e_ms, e2e_rids, _, _, _, e2e_steps = timed(host_io=True)
     scratch = from_scratch_prefill(w, plan, mk, flush, args, seed_base) if args.workload == "refill" else None
@@ -515,11 +563,9 @@ def run_kvm(args):
     # ---- CPU oracle sample (rank 0 only, single GPU runs only)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        secs, m = oracle_sample(w, 256)
-        cpu = {"value": m / secs, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
-               "sample": f"character 0, round 0: compaction + all {len(s.layer_kind)} layers for the first "
-                         f"{m} of {plan[0][3][0]} tail tokens (prefix {w.prefix_len[0]}), fp64 numpy, "
-                         f"{secs:.1f} s"}
+        secs, m, blocks = oracle_sample(w, oracle_state(w), CPU_BASELINE_TOKENS[args.workload])
+        cpu = {"value": m / (secs * blocks), "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+               "sample": sample_text(w, m, secs)}
     per_kernel = {}
     for name, d in kernels.items():
         per_kernel[name] = {"launches": d["launches"], "avg_us": 1e3 * d["total_ms"] / d["launches"],
@@ -528,10 +574,7 @@ def run_kvm(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": WORKLOAD_TEXT[args.workload], "name": args.workload, "chars": w.n_chars,
-                   "layers": len(s.layer_kind), "chain_rounds": R,
-                   "l2": "flushed before every step (256 MiB write), outside the timed events",
-                   "parallelism": f"{world} independent replica(s), characters per rank fixed"},
+        "config": workload_config(w, args, world),
         "roofline": roofline,
         "round_roofline": round_roofline,
         "cpu_baseline": cpu,
@@ -562,10 +605,10 @@ def run_kvm(args):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=64)
+    ap.add_argument("--steps", type=int, default=160)
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--impl", choices=["kvm", "reference"], default="kvm")
-    ap.add_argument("--workload", choices=list(WORKLOAD_TEXT), default="npc")
+    ap.add_argument("--workload", choices=list(WORKLOAD_TEXT), default="long")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:

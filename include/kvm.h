@@ -292,13 +292,21 @@ kvm_status kvm_update_round(kvm_ctx* ctx, const kvm_round* round, void* stream);
  * calls that may overlap on the GPU (other streams, other host threads on
  * the same device) race: order them.  A device-side wait that expires
  * (which valid arguments never cause) leaves that chunk unmoved and sets a
- * bit in the array's error word; this call does not read it back.
+ * bit in the array's error word; kvm_kv_compact_noalloc_check reads it.
  * Errors: KVM_E_INVAL, KVM_E_SPAN, KVM_E_CAPACITY, KVM_E_UNSUPPORTED,
  * KVM_E_CUDA. */
 kvm_status kvm_kv_compact_noalloc(void* K, void* V, int32_t* positions, int32_t n_slabs,
                                   int64_t slab_rows, int32_t head_dim, int32_t live,
                                   int32_t n_spans, const int32_t* span_begin,
                                   const int32_t* span_end, int32_t* new_live_out, void* stream);
+
+/* The failure signal of kvm_kv_compact_noalloc on the current device: waits
+ * for `stream`, then reads and clears the error word of the library's
+ * static scratch array.  Returns KVM_E_DEVICE if a call since the last check
+ * reported a bounds violation or an expired wait (the rows of that call are
+ * then undefined), KVM_OK otherwise.  Allocates nothing; the paper has no
+ * counterpart of this call.  Errors: KVM_E_DEVICE, KVM_E_CUDA. */
+kvm_status kvm_kv_compact_noalloc_check(void* stream);
 
 /* Copy the whole state of `src` into `dst`: every character's live KV,
  * positions, recurrent states, live lengths and cursors (§4.2: task-specific
@@ -326,6 +334,17 @@ kvm_status kvm_profile_read(kvm_ctx* ctx, int32_t kernel, int64_t* launches, dou
  * (and clears the word) if a kernel reported a violation since the last
  * check. */
 kvm_status kvm_check(kvm_ctx* ctx, void* stream);
+
+/* Failure-detection hook of the compaction's bounded waits (no paper
+ * counterpart).  polls: how many times a compaction block polls an earlier
+ * chunk's read flag before it gives up (0 restores the default, ~0.3-1 s).
+ * stall != 0: every block of later compactions of this context also waits
+ * on a device word that nothing sets, so each gives up after `polls` polls,
+ * moves nothing and reports an expired wait, which kvm_check returns as
+ * KVM_E_DEVICE (the context's caches are then undefined: restore them, e.g.
+ * with kvm_fork from a root).  Tests use it to exercise the failure path
+ * without a fault.  Errors: KVM_E_INVAL. */
+kvm_status kvm_debug_compact_wait(kvm_ctx* ctx, int32_t polls, int32_t stall);
 
 /* Number of kernel launches the library has enqueued since creation
  * (diagnostics for the benchmark). */

@@ -17,14 +17,13 @@
 // holds).  Blocks wait only on chunks with earlier tickets, which are
 // resident or finished, so the waits always end; each wait is still bounded
 // and reports kErrWait instead of spinning forever.
+#include <cstdio>
 #include <cstring>
 
 #include "kvm_internal.cuh"
 
 namespace kvm {
 namespace {
-
-constexpr int kWaitLimit = 1 << 22;   // ~0.3-1 s with the back-off below
 
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
     uint32_t v;
@@ -130,7 +129,14 @@ kv_compact_kernel(const __grid_constant__ CompactParams p) {
         for (int e = e_min + tid; e < chunk && !fail; e += 32) {
             int it = 0;
             while (ld_acquire(p.flags + (int64_t)(flag_base + e) * p.flag_stride) != p.epoch) {
-                if (++it > kWaitLimit) { fail = true; break; }
+                if (++it > p.wait_limit) { fail = true; break; }
+                __nanosleep(64);
+            }
+        }
+        if (p.never_set && tid == 0) {
+            int it = 0;
+            while (ld_acquire(p.never_set) != p.epoch) {
+                if (++it > p.wait_limit) { fail = true; break; }
                 __nanosleep(64);
             }
         }
@@ -306,6 +312,7 @@ extern "C" kvm_status kvm_kv_compact_noalloc(void* K, void* V, int32_t* position
     p.flags = flags;
     p.flag_stride = 1;
     p.err = reinterpret_cast<int32_t*>(scratch);
+    p.wait_limit = kCompactWaitLimit;
     CompactChar& c = p.ch[0];
     c.L_new = L_new;
     c.first = span_begin[0];
@@ -321,4 +328,26 @@ extern "C" kvm_status kvm_kv_compact_noalloc(void* K, void* V, int32_t* position
     e = cudaGetLastError();
     if (e != cudaSuccess) return report_error(KVM_E_CUDA, "kv_compact_noalloc: kernel launch failed");
     return KVM_OK;
+}
+
+extern "C" kvm_status kvm_kv_compact_noalloc_check(void* stream) {
+    using namespace kvm;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return report_error(KVM_E_CUDA, "kv_compact_noalloc_check: no usable current device");
+    // no call on this device yet: nothing can have failed
+    if (!g_noalloc_addr[dev]) return KVM_OK;
+    e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return report_error(KVM_E_CUDA, "kv_compact_noalloc_check: stream synchronize failed");
+    uint32_t word = 0;
+    e = cudaMemcpy(&word, g_noalloc_addr[dev], sizeof word, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return report_error(KVM_E_CUDA, "kv_compact_noalloc_check: reading the error word failed");
+    if (!word) return KVM_OK;
+    e = cudaMemset(g_noalloc_addr[dev], 0, sizeof word);
+    if (e != cudaSuccess) return report_error(KVM_E_CUDA, "kv_compact_noalloc_check: clearing the error word failed");
+    char msg[160];
+    snprintf(msg, sizeof msg, "kv_compact_noalloc: device error word 0x%x (%s%s); the rows of the failed call are undefined",
+             word, (word & kErrBounds) ? "bounds " : "", (word & kErrWait) ? "wait-timeout" : "");
+    return report_error(KVM_E_DEVICE, msg);
 }

@@ -112,6 +112,8 @@ struct kvm_ctx {
     CUtensorMap tmap_k, tmap_v;           // TMA maps of K, V (attention layers only)
     int64_t launches = 0;
     int rows_kv = 0, rows_pos = 0;
+    int compact_wait_limit = kCompactWaitLimit;   // polls of a compaction read flag before giving up
+    bool compact_stall = false;                   // failure-detection tests: wait on a word nothing sets
     // per-kernel timing (kvm_profile_*)
     bool prof = false;
     std::vector<cudaEvent_t> ev;          // 2 per timed launch
@@ -688,6 +690,10 @@ kvm_status launch_compaction(kvm_ctx* c, const SpanPlan& pl, cudaStream_t s, int
         p.flags = c->flags;
         p.flag_stride = kFlagStride;
         p.err = c->err;
+        p.wait_limit = c->compact_wait_limit;
+        // diag[15] is never written by any kernel (kvm_check clears it to 0,
+        // and epochs start at 1), so a wait on it can only expire
+        p.never_set = c->compact_stall ? reinterpret_cast<const uint32_t*>(c->diag + 15) : nullptr;
         int blk = 0;
         for (int b = 0; b < c->B; ++b) {
             CompactChar& ch = p.ch[b];
@@ -977,6 +983,7 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
             if (pl.L_new[b] + m > c->cap[b])
                 return fail(KVM_E_CAPACITY, "character %d: live %d + tail %d exceeds capacity %d", b, pl.L_new[b],
                             m, c->cap[b]);
+            if (c->cursor[b] + m > INT32_MAX) return fail(KVM_E_CAPACITY, "character %d: position ids overflow", b);
         }
         for (int l = 0; l < c->n_layers; ++l) {
             if (total > 0 && (!r->q[l] || !r->k[l] || !r->v[l] || !r->out[l]))
@@ -1128,6 +1135,14 @@ extern "C" kvm_status kvm_check(kvm_ctx* c, void* stream) {
         return fail(KVM_E_DEVICE, "device error word 0x%x (%s%s); first expired wait: block %d, tag 0x%x, parity %d",
                     e, (e & kErrBounds) ? "bounds " : "", (e & kErrWait) ? "wait-timeout" : "", d[0] - 1, d[1], d[2]);
     }
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_debug_compact_wait(kvm_ctx* c, int32_t polls, int32_t stall) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (polls < 0) return fail(KVM_E_INVAL, "polls must be >= 0");
+    c->compact_wait_limit = polls ? polls : kCompactWaitLimit;
+    c->compact_stall = stall != 0;
     return KVM_OK;
 }
 

@@ -48,6 +48,7 @@ constexpr int kErrWait = 2;         // a bounded wait expired
 constexpr int kCompactThreads = 256;
 constexpr int kCompactVecPerThread = 4;            // 16-byte vectors held per thread
 constexpr int kCompactVecPerChunk = kCompactThreads * kCompactVecPerThread;
+constexpr int kCompactWaitLimit = 1 << 22;        // default polls of a read flag (~0.3-1 s with the back-off)
 
 struct CompactChar {
     int32_t L_new;        // live length after removal
@@ -77,6 +78,10 @@ struct CompactParams {
     uint32_t* flags;      // read flag of chunk i at flags[i * flag_stride]
     int32_t flag_stride;  // 32 keeps every flag in its own 128-byte line (no line shared by pollers)
     int32_t* err;
+    int32_t wait_limit;   // polls of a read flag before the wait gives up (kErrWait)
+    // failure-detection test only: when set, every block also waits on this
+    // word, which nothing ever sets, so its wait expires after wait_limit polls
+    const uint32_t* never_set;
     CompactChar ch[kMaxChars];
     // segment k of a character: survivors whose new index is >= seg_start[k]
     // (and below the next segment's start) come from new index + seg_shift[k]

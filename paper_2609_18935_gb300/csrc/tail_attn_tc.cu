@@ -3,8 +3,10 @@
 //
 // Query tiles have 128 rows = (tail token, query head of one GQA group) pairs,
 // token-major, so each K/V tile serves all g heads of the group.  The work is
-// the list of (query tile, 64-key tile) units; it is cut into equal contiguous
-// ranges, one per persistent block (stream-K).  A block's range covers whole
+// the list of (query tile, 64-key tile) units; it is cut into contiguous
+// ranges, one per persistent block (stream-K), balanced by a cost model that
+// charges each unit 1 and each segment a block starts 8 more (the host
+// planner bisects for the smallest per-block cost).  A block's range covers whole
 // query tiles, whose outputs it normalises and stores directly, and at most
 // one partial tile at each end, whose unnormalised accumulator goes to a
 // workspace slot (2c for block c's first segment, 2c + 1 for its last) for

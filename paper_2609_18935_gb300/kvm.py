@@ -84,6 +84,8 @@ _SIGS = {
     "kvm_kv_compact_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int64, C.c_int32,
                                          C.c_int32, C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32),
                                          C.POINTER(C.c_int32), C.c_void_p]),
+    "kvm_kv_compact_noalloc_check": (C.c_int, [C.c_void_p]),
+    "kvm_debug_compact_wait": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
     "kvm_profile_enable": (C.c_int, [C.c_void_p, C.c_int32]),
     "kvm_profile_read": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double),
                                    C.c_int32]),
@@ -153,13 +155,33 @@ def kv_compact_noalloc(K, V, positions, live, span_begin, span_end, stream=None)
     int32 [slab_rows] or None.  Returns the new live length."""
     import torch
     load_library()
+    if K.dim() != 3:
+        raise ValueError("K must be [n_slabs][slab_rows][head_dim]")
     n_slabs, rows, D = K.shape
+    if tuple(V.shape) != tuple(K.shape):
+        raise ValueError(f"V has shape {tuple(V.shape)}, K has {tuple(K.shape)}")
+    dev = torch.cuda.current_device()
+    for name, t in (("K", K), ("V", V), ("positions", positions)):
+        if t is not None and (not t.is_cuda or t.device.index != dev):
+            raise ValueError(f"{name} must live on the current CUDA device (cuda:{dev})")
+    if positions is not None and positions.numel() < rows:
+        raise ValueError(f"positions holds {positions.numel()} entries, need >= slab_rows = {rows}")
     sb, se = _i32(span_begin), _i32(span_end)
+    if len(sb) != len(se):
+        raise ValueError("span_begin and span_end differ in length")
     new_live = C.c_int32()
     _check(_lib.kvm_kv_compact_noalloc(_dptr(K, torch.bfloat16), _dptr(V, torch.bfloat16),
                                        _dptr(positions, torch.int32), n_slabs, rows, D, int(live), len(sb),
                                        _p32(sb), _p32(se), C.byref(new_live), _stream(stream)))
     return new_live.value
+
+
+def kv_compact_noalloc_check(stream=None):
+    """kvm_kv_compact_noalloc_check: raise KvmError (KVM_E_DEVICE) if an
+    allocation-free compaction on the current device reported a failure
+    since the last check (the check clears it)."""
+    load_library()
+    _check(_lib.kvm_kv_compact_noalloc_check(_stream(stream)))
 
 
 def plan_removal(live, span_cu, span_begin, span_end):
@@ -356,6 +378,12 @@ class Context:
 
     def check(self, stream=None):
         _check(_lib.kvm_check(self._h, _stream(stream)))
+
+    def debug_compact_wait(self, polls=0, stall=False):
+        """kvm_debug_compact_wait: compaction wait limit (0 = default) and the
+        failure-detection stall (every later compaction block waits on a word
+        nothing sets and gives up after `polls` polls)."""
+        _check(_lib.kvm_debug_compact_wait(self._h, int(polls), int(bool(stall))))
 
     def launch_count(self) -> int:
         return int(_lib.kvm_launch_count(self._h))

@@ -188,15 +188,19 @@ class Pair:
                     assert np.array_equal(p1, new.caches[l].pos.astype(np.int32))
                     # appended rotated keys and values against the oracle's fp64 ones
                     if t1 > t0:
-                        key = ("append_k", l)
-                        errs[key] = max(errs.get(key, 0.0), rel_l2(O.bf16_to_f64(k1[:, L_new:]),
-                                                                  new.caches[l].K[:, L_new:]))
+                        errs[("append_k", l, b)] = rel_l2(O.bf16_to_f64(k1[:, L_new:]), new.caches[l].K[:, L_new:])
                         assert np.array_equal(O.bf16_to_f64(v1[:, L_new:]), new.caches[l].V[:, L_new:])
+        # the bar holds per (layer, character) for outputs and per (layer,
+        # character, head) for states, so that one wrong character or head
+        # cannot hide under the others' norm
         for l in dev_out:
-            if total > 0:
-                errs[("out", l)] = rel_l2(gpu_out[l], ora_out[l])
+            for b in range(B):
+                t0, t1 = tail_cu[b], tail_cu[b + 1]
+                if t1 > t0:
+                    errs[("out", l, b)] = rel_l2(gpu_out[l][t0:t1], ora_out[l][t0:t1])
         for l in s.gdn_layers:
             S_gpu = self.ctx.get_state(l).cpu().numpy().astype(np.float64)
-            S_ref = np.stack([self.oracle[b].states[l] for b in range(B)])
-            errs[("S", l)] = rel_l2(S_gpu, S_ref)
+            for b in range(B):
+                for h in range(s.n_gdn_heads):
+                    errs[("S", l, b, h)] = rel_l2(S_gpu[b, h], self.oracle[b].states[l][h])
         return errs

@@ -182,14 +182,27 @@ def test_population_full_size_round():
 def test_refill_equivalence_full_size():
     """refill: with nothing removed, a 512-token tail update on a 16384-token
     prefix equals the last 512 rows of a from-scratch prefill of 16896 tokens
-    (outputs, final states, cache bytes), both computed on the GPU."""
+    (outputs, final states, cache bytes), both computed on the GPU; and both
+    arms match the fp64 oracle run over the whole 16896-token sequence from an
+    empty state: attention rows of sampled tail tokens (every head) over the
+    full cache, and sampled delta-rule heads token by token from zero
+    (outputs of the tail and the final state)."""
     import torch
-    from harness import torch_bf16_bits, torch_bf16_to_f64, rel_l2
+    from harness import to_torch_bf16, torch_bf16_bits, torch_bf16_to_f64, rel_l2
+    from oracle import kvm_oracle as O
     from paper_2609_18935_gb300 import kvm
     w = W.make_workload("refill")
     s = w.shape
     N, M = 16384, 512
+    check_attn, check_gdn, heads = 3, 0, [0, 9]
     ins = W.device_round_inputs(w, 424242, [N + M])
+    host = W.tail_inputs(w, 0, [N + M], layers=[check_gdn, check_attn])   # the layers the oracle checks
+    for l, x in host.items():
+        d = {k: to_torch_bf16(x[k]).cuda() for k in ("q", "k", "v")}
+        if s.layer_kind[l] == W.GDN:
+            d["alpha"] = torch.from_numpy(x["alpha"]).cuda()
+            d["beta"] = torch.from_numpy(x["beta"]).cuda()
+        ins[l] = d
     mk = lambda mt: kvm.Context(s.layer_kind, s.n_q_heads, s.n_kv_heads, s.head_dim, s.rotary_dim,
                                 s.rope_theta, s.n_gdn_heads, s.d_k, s.d_v, [N + M], mt)
     shape = lambda l, T: (T, s.n_q_heads, s.head_dim) if s.layer_kind[l] == W.ATTN else (T, s.n_gdn_heads, s.d_v)
@@ -220,3 +233,29 @@ def test_refill_equivalence_full_size():
             assert np.array_equal(torch_bf16_bits(ka), torch_bf16_bits(kb))
             assert np.array_equal(torch_bf16_bits(va), torch_bf16_bits(vb))
     assert tail.get_live(0) == full.get_live(0) == (N + M, N + M)
+    # ---- the oracle over the whole sequence from an empty state
+    errs = {}
+    x = host[check_attn]
+    positions = np.arange(N + M)
+    krot = O.rope(O.bf16_to_f64(x["k"]), positions, s.rotary_dim, s.rope_theta)
+    vv = O.bf16_to_f64(x["v"])
+    g = s.n_q_heads // s.n_kv_heads
+    toks = sorted(set([0, 1, M - 1] + [int(t) for t in np.random.default_rng(12).integers(0, M, 5)]))
+    got_tail, got_full = torch_bf16_to_f64(o_tail[check_attn]), torch_bf16_to_f64(o_full[check_attn][N:])
+    for t in toks:
+        qrot = O.rope(O.bf16_to_f64(x["q"][N + t:N + t + 1]), positions[N + t:N + t + 1], s.rotary_dim, s.rope_theta)
+        ref = np.stack([O.attend_row(qrot[0, hq], krot[:N + t + 1, hq // g], vv[:N + t + 1, hq // g])
+                        for hq in range(s.n_q_heads)])
+        errs[("attn tail", t)] = rel_l2(got_tail[t], ref)
+        errs[("attn refill", t)] = rel_l2(got_full[t], ref)
+    x = host[check_gdn]
+    S_tail = tail.get_state(check_gdn).cpu().numpy().astype(np.float64)
+    got = torch_bf16_to_f64(o_tail[check_gdn])
+    for h in heads:
+        sl = np.s_[:, h:h + 1]
+        o, S = O.gdn_recurrent(O.bf16_to_f64(x["q"][sl]), O.bf16_to_f64(x["k"][sl]), O.bf16_to_f64(x["v"][sl]),
+                               O.f32_to_f64(x["alpha"][sl]), O.f32_to_f64(x["beta"][sl]),
+                               np.zeros((1, s.d_v, s.d_k)))
+        errs[("gdn tail out", h)] = rel_l2(got[:, h], o[N:, 0])
+        errs[("gdn S", h)] = rel_l2(S_tail[0, h], S[0])
+    _check(errs, "refill vs oracle")

@@ -29,6 +29,26 @@ def _unit(x):
     return x / np.linalg.norm(x, axis=-1, keepdims=True)
 
 
+# ---------------------------------------------------------------- input widening
+@pytest.mark.parametrize("bits,value", [
+    (0x3F80, 1.0), (0xC040, -3.0), (0x0000, 0.0), (0x4049, 3.140625), (0x3F81, 1.0 + 2.0 ** -7),
+    (0xBF00, -0.5), (0x7F7F, (2.0 - 2.0 ** -7) * 2.0 ** 127), (0x0080, 2.0 ** -126), (0x0001, 2.0 ** -133),
+    (0x7F80, math.inf), (0xFF80, -math.inf)])
+def test_bf16_widening_on_fixed_bit_patterns(bits, value):
+    """bf16 = sign | 8 exponent bits (bias 127) | 7 fraction bits: each bit
+    pattern's value written out by hand, including a subnormal and the
+    infinities."""
+    got = O.bf16_to_f64(np.array([bits], dtype=np.uint16))[0]
+    assert got == value
+    assert got.dtype == np.float64 if hasattr(got, "dtype") else True
+
+
+def test_bf16_widening_sign_of_zero_and_nan():
+    z = O.bf16_to_f64(np.array([0x8000], dtype=np.uint16))[0]
+    assert z == 0.0 and math.copysign(1.0, z) == -1.0
+    assert math.isnan(O.bf16_to_f64(np.array([0x7FC0], dtype=np.uint16))[0])
+
+
 # ---------------------------------------------------------------- golden
 def test_golden_gdn_hand_example():
     g = _gold("gdn_hand_2d.json")
