@@ -285,13 +285,18 @@ class CharacterState:
                               self.cursor)
 
 
-def tail_attn_prefill(cache: AttnCache, q, k_new, v_new, p: int, R: int, theta: float):
+def tail_attn_prefill(cache: AttnCache, q, k_new, v_new, p: int, R: int, theta: float, positions=None):
     """Append the tail's rotated keys and values at the true tail and attend.
 
     q [M][Hq][D], k_new/v_new [M][Hkv][D] (unrotated, fp64); tail token i has
-    position p + i.  Returns (out [M][Hq][D], new cache)."""
+    position p + i, or positions[i] when given (the placement variants of
+    §5.2: gapped or slot-preserving position ids).  Attention is causal in
+    processing order either way (every survivor and tail keys j <= i).
+    Returns (out [M][Hq][D], new cache)."""
     M = q.shape[0]
-    positions = p + np.arange(M, dtype=np.int64)
+    if positions is None:
+        positions = p + np.arange(M, dtype=np.int64)
+    positions = np.asarray(positions, dtype=np.int64)
     q_rot = rope(q, positions, R, theta)
     k_rot = rope(k_new, positions, R, theta)
     L_prev = cache.live
@@ -301,12 +306,34 @@ def tail_attn_prefill(cache: AttnCache, q, k_new, v_new, p: int, R: int, theta: 
     return out, AttnCache(K_all, V_all, np.concatenate([cache.pos, positions]))
 
 
+def rerotate_keys(cache: AttnCache, begin: int, end: int, new_pos, R: int, theta: float) -> AttnCache:
+    """Tail-and-relocate (§5.2): the stored keys of live entries [begin, end)
+    were rotated at cache.pos; turn them to new_pos.  A key rotated at p and
+    then by the angle of (q - p) is the key rotated at q, so each entry is
+    rotated by its (new - old) difference; values are untouched.  Returns a
+    new cache with the keys and positions replaced."""
+    out = cache.copy()
+    new_pos = np.asarray(new_pos, dtype=np.int64)
+    delta = new_pos - cache.pos[begin:end]
+    ks = np.transpose(cache.K[:, begin:end], (1, 0, 2))          # [n][Hkv][D]
+    out.K[:, begin:end] = np.transpose(rope(ks, delta, R, theta), (1, 0, 2))
+    out.pos[begin:end] = new_pos
+    return out
+
+
 def maintenance_round(state: CharacterState, layer_kind, begins, ends,
-                      inputs: dict, R: int, theta: float):
+                      inputs: dict, R: int, theta: float, positions=None, delimiters=None):
     """One round for one character: Eq. 2 on every attention layer, then
     Eq. 3 layer by layer in model order, then p += M.
 
     inputs[layer] = dict(q, k, v[, alpha, beta]) as fp64 arrays (tail only).
+    positions: optional [M] position ids of the tail (placement variants,
+    §5.2); the cursor then moves to max(p, largest id + 1).
+    delimiters: optional (begins, ends), half-open tail-index ranges of
+    maintenance delimiters (§4.2): processed with the tail, then their
+    direct KV are removed from every attention layer; their effect on the
+    recurrent states and on later tail tokens remains, and their position
+    ids stay consumed.
     Returns (outputs {layer: [M][heads][dim]}, new state).  `state` is not
     modified."""
     new = state.copy()
@@ -322,12 +349,24 @@ def maintenance_round(state: CharacterState, layer_kind, begins, ends,
         M = x["q"].shape[0]
         if kind == 1:
             outs[l], new.caches[l] = tail_attn_prefill(new.caches[l], x["q"], x["k"], x["v"],
-                                                       new.cursor, R, theta)
+                                                       new.cursor, R, theta, positions)
         else:
             outs[l], new.states[l] = gdn_recurrent(x["q"], x["k"], x["v"], x["alpha"],
                                                    x["beta"], new.states[l])
     if M is not None:
-        new.cursor += M
+        if positions is None:
+            new.cursor += M
+        elif M > 0:
+            new.cursor = max(new.cursor, int(np.max(positions)) + 1)
+    if delimiters is not None and len(delimiters[0]) > 0:
+        for l, kind in enumerate(layer_kind):
+            if kind == 1:
+                c = new.caches[l]
+                L_prev = c.live - M
+                db = [L_prev + int(x) for x in delimiters[0]]
+                de = [L_prev + int(x) for x in delimiters[1]]
+                K, V, pos, _ = kv_compact(c.K, c.V, c.pos, db, de)
+                new.caches[l] = AttnCache(K, V, pos)
     return outs, new
 
 

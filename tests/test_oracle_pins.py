@@ -429,3 +429,178 @@ def test_removal_leaves_recurrent_state_and_cursor_alone():
     r_outs, r = O.refill(st["layer_kind"], txt, *args)
     assert not np.allclose(r.states[0], a.states[0])
     assert not np.allclose(r_outs[1][-M:], o_a[1])
+
+
+# ---------------------------------------------------------------- placement variants (§5.2)
+def test_rerotation_round_trip_is_identity():
+    """Turning stored keys from p to q and back to p gives the keys back."""
+    D, R, theta = 16, 8, 1e4
+    n = 7
+    x = rng.standard_normal((n, 2, D))
+    p = rng.integers(0, 500_000, n)
+    q = rng.integers(0, 500_000, n)
+    cache = O.AttnCache(np.transpose(O.rope(x, p, R, theta), (1, 0, 2)), rng.standard_normal((2, n, D)), p)
+    there = O.rerotate_keys(cache, 0, n, q, R, theta)
+    back = O.rerotate_keys(there, 0, n, p, R, theta)
+    np.testing.assert_allclose(back.K, cache.K, atol=1e-9)
+    np.testing.assert_array_equal(back.V, cache.V)
+    np.testing.assert_array_equal(back.pos, p)
+    assert not np.allclose(there.K, cache.K)
+
+
+def test_rerotation_equals_rotation_at_the_target_position():
+    """A key stored at p, turned to q, equals the raw key rotated at q in
+    RoFormer's complex form (an independent statement of the rotation)."""
+    D, R, theta = 16, 8, 1e4
+    n = 5
+    x = rng.standard_normal((n, 2, D))
+    p = np.array([3, 90, 1000, 261_955, 479_547])
+    q = np.array([10_003, 2, 479_547, 20, 0])
+    cache = O.AttnCache(np.transpose(O.rope(x, p, R, theta), (1, 0, 2)), np.zeros((2, n, D)), p)
+    moved = O.rerotate_keys(cache, 1, 4, q[1:4], R, theta)
+    h = R // 2
+    for j in range(1, 4):
+        for kv in range(2):
+            for d in range(h):
+                w = theta ** (-(2 * d) / R)
+                z = complex(x[j, kv, d], x[j, kv, d + h]) * complex(math.cos(q[j] * w), math.sin(q[j] * w))
+                assert abs(moved.K[kv, j, d] - z.real) < 1e-8
+                assert abs(moved.K[kv, j, d + h] - z.imag) < 1e-8
+    np.testing.assert_array_equal(moved.K[:, [0, 4]], cache.K[:, [0, 4]])
+    assert list(moved.pos) == [3, 2, 479_547, 20, 479_547]
+
+
+def test_explicit_true_tail_positions_equal_the_default():
+    st = _stack()
+    N, M = 20, 7
+    ins = _tokens(N + M, st)
+    args = (st["Hkv"], st["D"], st["H"], st["dk"], st["dv"], st["R"], st["theta"])
+    _, pre = O.refill(st["layer_kind"], _cut(ins, 0, N), *args)
+    tail = _cut(ins, N, N + M)
+    o_a, a = O.maintenance_round(pre, st["layer_kind"], [2], [5], tail, st["R"], st["theta"])
+    o_b, b = O.maintenance_round(pre, st["layer_kind"], [2], [5], tail, st["R"], st["theta"],
+                                 positions=np.arange(N, N + M))
+    for l in o_a:
+        np.testing.assert_array_equal(o_a[l], o_b[l])
+    for l in a.caches:
+        np.testing.assert_array_equal(a.caches[l].K, b.caches[l].K)
+        np.testing.assert_array_equal(a.caches[l].pos, b.caches[l].pos)
+    assert a.cursor == b.cursor == N + M
+
+
+def test_gapped_prefill_brute_force():
+    """Fresh gapped prefill (§5.2): the text read from an empty state with
+    gaps between records' position ids.  Each output row is recomputed with
+    scalar loops: keys rotated in the complex form at their ids, causal in
+    reading order, softmax by hand."""
+    Hq, Hkv, D, R, theta = 4, 2, 8, 8, 1e4
+    pos = np.array([0, 1, 2, 10_000, 10_001, 20_000, 20_001, 20_002])
+    M = len(pos)
+    q = rng.standard_normal((M, Hq, D))
+    k = _unit(rng.standard_normal((M, Hkv, D)))
+    v = rng.standard_normal((M, Hkv, D))
+    empty = O.AttnCache(np.zeros((Hkv, 0, D)), np.zeros((Hkv, 0, D)), np.zeros(0, np.int64))
+    out, cache = O.tail_attn_prefill(empty, q, k, v, 0, R, theta, positions=pos)
+    h = R // 2
+
+    def rot(x, p):
+        y = list(x)
+        for d in range(h):
+            w = theta ** (-(2 * d) / R)
+            z = complex(x[d], x[d + h]) * complex(math.cos(p * w), math.sin(p * w))
+            y[d], y[d + h] = z.real, z.imag
+        return y
+
+    for i in range(M):
+        for hq in range(Hq):
+            kv = hq // (Hq // Hkv)
+            qi = rot(q[i, hq], pos[i])
+            sc = [sum(a * b for a, b in zip(qi, rot(k[j, kv], pos[j]))) / math.sqrt(D) for j in range(i + 1)]
+            mx = max(sc)
+            w = [math.exp(x - mx) for x in sc]
+            ref = [sum(w[j] * v[j, kv, d] for j in range(i + 1)) / sum(w) for d in range(D)]
+            np.testing.assert_allclose(out[i, hq], ref, atol=1e-10)
+    np.testing.assert_array_equal(cache.pos, pos)
+
+
+def test_slot_positions_change_attention_but_not_the_recurrence():
+    """Slot-preserving placement (§5.2) changes only the rotary ids of the
+    replacement: attention outputs differ from the true tail, the recurrent
+    layers (which carry no positions) do not; the cursor does not move past
+    the largest id used."""
+    st = _stack()
+    N, M = 30, 6
+    ins = _tokens(N + M, st)
+    args = (st["Hkv"], st["D"], st["H"], st["dk"], st["dv"], st["R"], st["theta"])
+    _, pre = O.refill(st["layer_kind"], _cut(ins, 0, N), *args)
+    tail = _cut(ins, N, N + M)
+    o_t, t = O.maintenance_round(pre, st["layer_kind"], [10], [16], tail, st["R"], st["theta"])
+    o_s, s = O.maintenance_round(pre, st["layer_kind"], [10], [16], tail, st["R"], st["theta"],
+                                 positions=np.arange(10, 16))
+    for l in t.states:
+        np.testing.assert_array_equal(t.states[l], s.states[l])
+        np.testing.assert_array_equal(o_t[l], o_s[l])
+    for l in t.caches:
+        assert not np.allclose(o_t[l], o_s[l])
+        assert list(s.caches[l].pos[-M:]) == list(range(10, 16))
+    assert t.cursor == N + M and s.cursor == N
+
+
+def test_relative_shift_invariance_with_explicit_positions():
+    """Shifting every id (the cache's rotation and the tail's) by the same
+    amount leaves attention outputs unchanged (relative positions only)."""
+    Hq, Hkv, D, R, theta = 4, 2, 16, 8, 1e4
+    L, M, shift = 9, 5, 123_457
+    kraw = _unit(rng.standard_normal((L, Hkv, D)))
+    vals = rng.standard_normal((Hkv, L, D))
+    cpos = np.array([0, 3, 4, 8, 20, 21, 22, 40, 41])
+    tpos = np.array([100, 7, 300, 301, 5])
+    q = rng.standard_normal((M, Hq, D))
+    k = _unit(rng.standard_normal((M, Hkv, D)))
+    v = rng.standard_normal((M, Hkv, D))
+    outs = []
+    for s in (0, shift):
+        cache = O.AttnCache(np.transpose(O.rope(kraw, cpos + s, R, theta), (1, 0, 2)), vals, cpos + s)
+        o, _ = O.tail_attn_prefill(cache, q, k, v, 0, R, theta, positions=tpos + s)
+        outs.append(o)
+    np.testing.assert_allclose(outs[0], outs[1], atol=1e-8)
+
+
+# ---------------------------------------------------------------- maintenance delimiters (§4.2)
+def test_delimiters_leave_no_kv_but_keep_their_effect():
+    st = _stack()
+    N, M = 25, 10
+    ins = _tokens(N + M, st)
+    args = (st["Hkv"], st["D"], st["H"], st["dk"], st["dv"], st["R"], st["theta"])
+    _, pre = O.refill(st["layer_kind"], _cut(ins, 0, N), *args)
+    tail = _cut(ins, N, N + M)
+    delim = ([0, 7], [2, 8])                     # tail tokens 0, 1 and 7 are delimiters
+    o_d, d = O.maintenance_round(pre, st["layer_kind"], [3], [6], tail, st["R"], st["theta"], delimiters=delim)
+    o_k, k = O.maintenance_round(pre, st["layer_kind"], [3], [6], tail, st["R"], st["theta"])
+    # the round itself is the same round: every output, every recurrent state
+    for l in o_d:
+        np.testing.assert_array_equal(o_d[l], o_k[l])
+    for l in d.states:
+        np.testing.assert_array_equal(d.states[l], k.states[l])
+    # their ids stay consumed; their KV are gone and nothing else is
+    assert d.cursor == k.cursor == N + M
+    keep = np.ones(N - 3 + M, bool)
+    keep[[N - 3 + 0, N - 3 + 1, N - 3 + 7]] = False
+    for l in d.caches:
+        assert d.caches[l].live == N - 3 + M - 3
+        np.testing.assert_array_equal(d.caches[l].K, k.caches[l].K[:, keep])
+        np.testing.assert_array_equal(d.caches[l].pos, k.caches[l].pos[keep])
+        assert N + 0 not in d.caches[l].pos and N + 7 not in d.caches[l].pos
+    # their indirect effect remains: without the delimiter tokens the state differs
+    plain = {l: {kk: np.delete(x, [0, 1, 7], axis=0) for kk, x in dd.items()} for l, dd in tail.items()}
+    _, nd = O.maintenance_round(pre, st["layer_kind"], [3], [6], plain, st["R"], st["theta"])
+    assert not np.allclose(nd.states[0], d.states[0])
+    # a later round attends over the cache without the delimiters' keys
+    nxt = _tokens(3, st)
+    o2, _ = O.maintenance_round(d, st["layer_kind"], [], [], nxt, st["R"], st["theta"])
+    c = d.caches[1]
+    qr = O.rope(nxt[1]["q"], np.arange(N + M, N + M + 3), st["R"], st["theta"])
+    kr = O.rope(nxt[1]["k"], np.arange(N + M, N + M + 3), st["R"], st["theta"])
+    keys = np.concatenate([c.K[0], kr[:1, 0]])
+    vals = np.concatenate([c.V[0], nxt[1]["v"][:1, 0]])
+    np.testing.assert_allclose(o2[1][0, 0], O.attend_row(qr[0, 0], keys, vals), atol=1e-12)
