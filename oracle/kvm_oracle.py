@@ -170,6 +170,68 @@ def tail_attention(q_rot, K_all, V_all, L_prev: int) -> np.ndarray:
 
 
 # ----------------------------------------------------------------------------
+# Attention-probe diagnostics (§5.3; Appendix C)
+# ----------------------------------------------------------------------------
+def probe_distributions(cache: AttnCache, q_raw) -> np.ndarray:
+    """Per probe query and head, the attention distribution over the live
+    entries.  The probe queries are those of the last n_q live entries:
+    q_raw [n_q][Hq][D] unrotated; query i sits at live index L - n_q + i,
+    is rotated at that entry's position by the caller-supplied rotation
+    (rotate_probe_queries) and sees entries 0 .. L - n_q + i.  Removed
+    records left no entries, so the softmax denominator runs over live
+    tokens only.  Returns [n_q][Hq][L], zero past each query's limit."""
+    q = np.asarray(q_raw, np.float64)
+    n_q, Hq, D = q.shape
+    Hkv = cache.K.shape[0]
+    g = Hq // Hkv
+    L = cache.live
+    out = np.zeros((n_q, Hq, L))
+    for i in range(n_q):
+        n_vis = L - n_q + i + 1
+        for h in range(Hq):
+            s = cache.K[h // g, :n_vis] @ q[i, h] / math.sqrt(D)
+            w = np.exp(s - s.max())
+            out[i, h, :n_vis] = w / w.sum()
+    return out
+
+
+def rotate_probe_queries(cache: AttnCache, q_raw, R: int, theta: float) -> np.ndarray:
+    """Rotate probe query i at the position of live entry L - n_q + i."""
+    n_q = np.asarray(q_raw).shape[0]
+    return rope(q_raw, cache.pos[cache.live - n_q:], R, theta)
+
+
+def attention_probe(cache: AttnCache, q_raw, R: int, theta: float) -> np.ndarray:
+    """The probe distribution over the live entries [L]: the per query and
+    head distributions averaged over the n_q queries and every head."""
+    d = probe_distributions(cache, rotate_probe_queries(cache, q_raw, R, theta))
+    return d.mean(axis=(0, 1))
+
+
+def group_mass(a, group_of, n_groups: int) -> np.ndarray:
+    """Summed probability of each group; entries with group -1 count for none."""
+    m = np.zeros(n_groups)
+    for x, gid in zip(np.asarray(a, np.float64), np.asarray(group_of)):
+        if gid >= 0:
+            m[int(gid)] += x
+    return m
+
+
+def effective_group_count(mass) -> float:
+    """exp(-sum_i a_i log a_i) for the group probabilities a_i = mass_i /
+    sum(mass) (0 log 0 = 0), the dispersion measure of §5.3."""
+    m = np.asarray(mass, np.float64)
+    a = m / m.sum()
+    nz = a[a > 0]
+    return float(np.exp(-(nz * np.log(nz)).sum()))
+
+
+def total_variation(p, q) -> float:
+    """Total variation distance 0.5 * sum |p_i - q_i| (§6.3)."""
+    return float(0.5 * np.abs(np.asarray(p, np.float64) - np.asarray(q, np.float64)).sum())
+
+
+# ----------------------------------------------------------------------------
 # Gated delta rule (§4.1, Gated DeltaNet)
 # ----------------------------------------------------------------------------
 def gdn_recurrent(q, k, v, alpha, beta, S0):

@@ -604,3 +604,95 @@ def test_delimiters_leave_no_kv_but_keep_their_effect():
     keys = np.concatenate([c.K[0], kr[:1, 0]])
     vals = np.concatenate([c.V[0], nxt[1]["v"][:1, 0]])
     np.testing.assert_allclose(o2[1][0, 0], O.attend_row(qr[0, 0], keys, vals), atol=1e-12)
+
+
+# ---------------------------------------------------------------- attention probes (§5.3)
+def _probe_cache(L=23, Hkv=2, D=16, R=8, theta=1e4):
+    pos = np.sort(rng.choice(np.arange(1000), size=L, replace=False))
+    kraw = _unit(rng.standard_normal((L, Hkv, D)))
+    K = np.transpose(O.rope(kraw, pos, R, theta), (1, 0, 2))
+    return O.AttnCache(K, rng.standard_normal((Hkv, L, D)), pos)
+
+
+def test_probe_rows_are_the_attention_weights():
+    """Each probe row sums to 1 over the keys its query sees, and weighting
+    the values by it reproduces the attention output of that query (the
+    reference softmax reconstructs the attention)."""
+    c = _probe_cache()
+    n_q, Hq = 5, 4
+    q = rng.standard_normal((n_q, Hq, 16))
+    qr = O.rotate_probe_queries(c, q, 8, 1e4)
+    d = O.probe_distributions(c, qr)
+    np.testing.assert_allclose(d.sum(axis=2), 1.0, atol=1e-12)
+    for i in range(n_q):
+        lim = c.live - n_q + i + 1
+        assert np.all(d[i, :, lim:] == 0)
+        for h in range(Hq):
+            kv = h // 2
+            np.testing.assert_allclose(d[i, h] @ c.V[kv], O.attend_row(qr[i, h], c.K[kv, :lim], c.V[kv, :lim]),
+                                       atol=1e-12)
+    a = O.attention_probe(c, q, 8, 1e4)
+    assert abs(a.sum() - 1.0) < 1e-12
+
+
+def test_probe_holes_excluded_equals_masking():
+    """Probe over the compacted cache = probe over the cache before removal
+    with the removed keys' scores at -inf (scipy softmax), renumbered."""
+    c = _probe_cache(L=30)
+    n_q, Hq = 4, 4
+    q = rng.standard_normal((n_q, Hq, 16))
+    K, V, pos, gather = O.kv_compact(c.K, c.V, c.pos, [3, 12], [7, 20])
+    cc = O.AttnCache(K, V, pos)
+    got = O.probe_distributions(cc, O.rotate_probe_queries(cc, q, 8, 1e4))
+    qr = O.rope(q, pos[-n_q:], 8, 1e4)
+    keep = O.keep_mask(30, [3, 12], [7, 20])
+    for i in range(n_q):
+        lim_old = gather[cc.live - n_q + i] + 1
+        for h in range(Hq):
+            sc = c.K[h // 2, :lim_old] @ qr[i, h] / 4.0
+            sc = np.where(keep[:lim_old], sc, -np.inf)
+            ref = softmax(sc)
+            np.testing.assert_allclose(got[i, h, :cc.live - n_q + i + 1], ref[keep[:lim_old]], atol=1e-12)
+
+
+def test_probe_brute_force_tiny():
+    c = _probe_cache(L=6, Hkv=1, D=4, R=4)
+    q = rng.standard_normal((2, 2, 4))
+    qr = O.rotate_probe_queries(c, q, 4, 1e4)
+    got = O.attention_probe(c, q, 4, 1e4)
+    acc = [0.0] * 6
+    for i in range(2):
+        for h in range(2):
+            lim = 6 - 2 + i + 1
+            sc = [sum(qr[i, h, d] * c.K[0, j, d] for d in range(4)) / 2.0 for j in range(lim)]
+            mx = max(sc)
+            w = [math.exp(x - mx) for x in sc]
+            for j in range(lim):
+                acc[j] += w[j] / sum(w) / 4
+    np.testing.assert_allclose(got, acc, atol=1e-12)
+
+
+def test_effective_group_count_closed_forms():
+    for n in (1, 2, 7, 34):
+        assert abs(O.effective_group_count(np.ones(n)) - n) < 1e-12
+        assert abs(O.effective_group_count(np.full(n, 0.37)) - n) < 1e-12      # scale-free
+    assert abs(O.effective_group_count([0, 0, 5.0, 0]) - 1.0) < 1e-12
+    p = 0.2
+    assert abs(O.effective_group_count([p, 1 - p]) - math.exp(-(p * math.log(p) + (1 - p) * math.log(1 - p)))) < 1e-12
+    m = O.group_mass([0.1, 0.2, 0.3, 0.4], [0, -1, 0, 2], 3)
+    np.testing.assert_allclose(m, [0.4, 0.0, 0.4])
+
+
+def test_total_variation_is_the_largest_event_difference():
+    """TVD = max over events A of |P(A) - Q(A)| (its definition as a
+    supremum), checked by enumerating every subset of a small support."""
+    import itertools
+    for _ in range(20):
+        p = rng.random(6)
+        p /= p.sum()
+        q = rng.random(6)
+        q /= q.sum()
+        best = max(abs(sum(p[list(A)]) - sum(q[list(A)])) for r in range(7) for A in itertools.combinations(range(6), r))
+        assert abs(O.total_variation(p, q) - best) < 1e-12
+    assert O.total_variation([1, 0], [0, 1]) == 1.0
+    assert O.total_variation([0.3, 0.7], [0.3, 0.7]) == 0.0
