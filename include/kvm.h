@@ -80,6 +80,14 @@ typedef struct kvm_model_desc {
     int32_t n_gdn_heads;
     int32_t d_k;
     int32_t d_v;
+    /* Short convolution of the delta-rule layers (§4.1: R_t holds the
+     * recurrent and the convolution states): 0 = none (q, k, v are used as
+     * given); 4 = the layer's q, k, v inputs are pre-convolution projections,
+     * filtered per channel by a causal depthwise convolution of width 4 over
+     * the tail and the last three inputs of earlier rounds (the carried conv
+     * state), then SiLU; k is then scaled to unit L2 norm per head.  Weights
+     * per layer with kvm_set_conv_weights. */
+    int32_t conv_kernel;
 } kvm_model_desc;
 
 /* ---------------------------------------------------------------- lifetime */
@@ -126,6 +134,18 @@ kvm_status kvm_get_positions(kvm_ctx* ctx, int32_t b, int32_t* pos_out, void* st
 kvm_status kvm_set_state(kvm_ctx* ctx, int32_t layer, const float* S, void* stream);
 kvm_status kvm_get_state(kvm_ctx* ctx, int32_t layer, float* S_out, void* stream);
 
+/* Short-convolution weights and state of delta-rule layer `layer` (model
+ * index), for contexts created with conv_kernel = 4.  Channels are ordered q
+ * [H][d_k], k [H][d_k], v [H][d_v] (C = H (2 d_k + d_v)).
+ * kvm_set_conv_weights: w device fp32 [C][4], tap i multiplies the input
+ * 3 - i tokens back (tap 3 is the current token); the context keeps a copy.
+ * kvm_get_conv_state / kvm_set_conv_state: device bf16 [n_chars][3][C], the
+ * last three pre-convolution inputs of each character (oldest first); a new
+ * context starts from zeros.  Errors: KVM_E_INVAL (no conv, wrong layer). */
+kvm_status kvm_set_conv_weights(kvm_ctx* ctx, int32_t layer, const float* w, void* stream);
+kvm_status kvm_get_conv_state(kvm_ctx* ctx, int32_t layer, void* state_out, void* stream);
+kvm_status kvm_set_conv_state(kvm_ctx* ctx, int32_t layer, const void* state, void* stream);
+
 /* Host view of character b's live length and cursor (no synchronization). */
 kvm_status kvm_get_live(kvm_ctx* ctx, int32_t b, int32_t* live, int64_t* cursor);
 
@@ -133,7 +153,10 @@ kvm_status kvm_get_live(kvm_ctx* ctx, int32_t b, int32_t* live, int64_t* cursor)
  * live-index spans, checking each against the live entries (§4.2: deletion
  * ranges are verified against live spans).  A range must cover at least one
  * live entry and every live entry whose position lies in it; the ranges
- * must be sorted and disjoint.  Outputs host [n].  Errors: KVM_E_SPAN. */
+ * must be sorted and disjoint.  When per-token positions or re-rotation have
+ * left the live positions out of order, the entries a range covers must form
+ * one contiguous run of live indices.  Outputs host [n].  Errors:
+ * KVM_E_SPAN. */
 kvm_status kvm_spans_from_positions(kvm_ctx* ctx, int32_t b, int32_t n,
                                     const int64_t* pos_begin, const int64_t* pos_end,
                                     int32_t* span_begin, int32_t* span_end);
@@ -156,7 +179,7 @@ kvm_status kvm_plan_removal(int32_t n_chars, const int32_t* live, const int32_t*
                             int32_t* first_moved);
 
 /* kvm_spans_from_positions on a caller's copy of one character's live
- * positions: positions host [live], strictly increasing.  Same mapping,
+ * positions: positions host [live], non-negative, in live order.  Same mapping,
  * checks and errors (KVM_E_INVAL for bad arguments, KVM_E_SPAN for ranges). */
 kvm_status kvm_plan_spans_from_positions(int32_t live, const int32_t* positions, int32_t n,
                                          const int64_t* pos_begin, const int64_t* pos_end,
@@ -213,7 +236,8 @@ kvm_status kvm_tail_attn_prefill(kvm_ctx* ctx, int32_t layer, const int32_t* tai
                                  void* out, void* stream);
 
 /* Eq. 3 for one gated-delta-rule layer (model index `layer`): advance each
- * character's carried state S through its M_b tail tokens,
+ * character's carried state S (and, with conv_kernel = 4, first its conv
+ * state over the q/k/v inputs, see kvm_model_desc) through its M_b tail tokens,
  *   S_t = alpha_t S_{t-1} (I - beta_t k_t k_t^T) + beta_t v_t k_t^T,
  *   o_t = S_t q_t,
  * computed in chunks of 64 tokens (WY/UT form) starting at the first tail
@@ -231,6 +255,36 @@ kvm_status kvm_gdn_chunk_scan_from_state(kvm_ctx* ctx, int32_t layer, const int3
  * (host bookkeeping; the device positions were written by the attention
  * layers).  tail_cu host [n_chars+1]. */
 kvm_status kvm_advance(kvm_ctx* ctx, const int32_t* tail_cu);
+
+/* Placement variants of the tail (§5.2: fresh gapped prefill reads the text
+ * with gaps between records' position ids; slot-preserving maintenance
+ * rotates the replacement's queries and keys at its original slot's ids).
+ * As kvm_tail_attn_prefill, but tail token n (packed) is rotated at, and
+ * stored with, position id tail_pos[n] (host [sum M], each >= 0; NULL = the
+ * true tail p_b + i).  Attention stays causal in processing order: a tail
+ * token sees every surviving entry and the tail tokens before it, whatever
+ * their ids.  Errors: as kvm_tail_attn_prefill. */
+kvm_status kvm_tail_attn_prefill_at(kvm_ctx* ctx, int32_t layer, const int32_t* tail_cu,
+                                    const int32_t* tail_pos, const void* q, const void* k_new,
+                                    const void* v_new, void* out, void* stream);
+
+/* kvm_advance after kvm_tail_attn_prefill_at: the host position mirror gets
+ * tail_pos (host [sum M], NULL = p_b + i) and the cursor moves to
+ * max(p_b, largest position + 1), so ids are never reused. */
+kvm_status kvm_advance_at(kvm_ctx* ctx, const int32_t* tail_cu, const int32_t* tail_pos);
+
+/* Tail-and-relocate (§5.2, §6.3): after a tail computed at tail positions,
+ * turn the stored keys of character b's live entries [live_begin, live_end)
+ * in every attention layer from the positions they were rotated at to
+ * new_pos (host [live_end - live_begin], each >= 0): each rotary pair of a
+ * key is rotated by (new_pos - old position) * omega_d, which for rotations
+ * equals rotating the unrotated key at new_pos.  Values, recurrent states
+ * and the entries' order are unchanged; the stored positions become new_pos
+ * and the cursor moves to max(p_b, largest new position + 1).  The keys are
+ * re-rounded to bf16 once.  Errors: KVM_E_INVAL, KVM_E_SPAN (range outside
+ * the live entries). */
+kvm_status kvm_rerotate_keys(kvm_ctx* ctx, int32_t b, int32_t live_begin, int32_t live_end,
+                             const int32_t* new_pos, void* stream);
 
 /* One whole maintenance round (Eq. 2 then Eq. 3 for every layer; §4.1, §4.2):
  * kv_compact, then every layer in model order (tail_attn_prefill or
@@ -263,6 +317,23 @@ typedef struct kvm_round {
     void* const* out;              /* [n_layers] */
     int32_t io_on_host;
     int32_t* gather_out;           /* optional device, see kvm_kv_compact */
+    /* Placement variants (§5.2), optional: tail_pos host [sum M] gives each
+     * tail token its position id (>= 0) for RoPE and for the stored
+     * position; NULL places the tail at the true tail p_b + i.  Attention
+     * stays causal in processing order: a tail token sees every surviving
+     * entry and the tail tokens before it, whatever their position ids.
+     * With tail_pos the cursor moves to max(p_b, largest position + 1). */
+    const int32_t* tail_pos;
+    /* Maintenance delimiters (§4.2), optional: delim_cu host [n_chars+1]
+     * offsets into delim_begin/delim_end (host), half-open tail-index ranges
+     * [s, e) within [0, M_b), sorted and disjoint per character.  Those tail
+     * tokens are processed like the rest (later tail tokens attend to them,
+     * the recurrent states absorb them), then their KV leave every attention
+     * layer at the end of the round; their position ids stay consumed.
+     * NULL: no delimiters. */
+    const int32_t* delim_cu;
+    const int32_t* delim_begin;
+    const int32_t* delim_end;
 } kvm_round;
 
 kvm_status kvm_update_round(kvm_ctx* ctx, const kvm_round* round, void* stream);
@@ -308,6 +379,39 @@ kvm_status kvm_kv_compact_noalloc(void* K, void* V, int32_t* positions, int32_t 
  * counterpart of this call.  Errors: KVM_E_DEVICE, KVM_E_CUDA. */
 kvm_status kvm_kv_compact_noalloc_check(void* stream);
 
+/* ------------------------------------------------------------ diagnostics */
+
+/* Attention probe (§5.3; Appendix C): how the last n_q query tokens of
+ * character b distribute attention over its live KV in attention layer
+ * `layer` (model index), reconstructed with a float32 reference softmax.
+ * q: device [n_q][n_q_heads][D] bf16, the unrotated queries of the last n_q
+ * live entries (the probe tokens, already appended by a round); query i is
+ * rotated at the position of live entry L - n_q + i and sees live entries
+ * 0 .. L - n_q + i (causal in processing order).  Removed records leave no
+ * entries, so the denominator runs over live tokens only (holes excluded).
+ * probs_out: device fp32 [L] (L = live length), the probability of each live
+ * entry averaged over the n_q queries and all query heads (sums to 1).
+ * group_of: optional device int32 [L], a group id in [0, n_groups) per live
+ * entry (-1: in no group), e.g. the memory record it belongs to;
+ * group_mass_out: device fp32 [n_groups], the summed probability per group.
+ * 1 <= n_q <= min(16, L).  Uses the context's workspace; enqueued on
+ * `stream`.  Errors: KVM_E_INVAL.  A group id >= n_groups is reported by
+ * kvm_check (KVM_E_DEVICE). */
+kvm_status kvm_attn_probe(kvm_ctx* ctx, int32_t layer, int32_t b, int32_t n_q, const void* q,
+                          float* probs_out, const int32_t* group_of, int32_t n_groups,
+                          float* group_mass_out, void* stream);
+
+/* Effective group count (§5.3): exp(-sum_i a_i log a_i) for the group
+ * probabilities a_i = mass_i / sum(mass) (0 log 0 = 0) -- a dispersion
+ * measure: n for a uniform spread over n groups, 1 for a single group.
+ * mass host [n_groups], non-negative, not all zero; *out host.  Host only.
+ * Errors: KVM_E_INVAL. */
+kvm_status kvm_effective_group_count(int32_t n_groups, const double* mass, double* out);
+
+/* Total variation distance between two distributions over the same n
+ * entries (§6.3): 0.5 * sum_i |p_i - q_i|.  Host only.  Errors: KVM_E_INVAL. */
+kvm_status kvm_total_variation(int32_t n, const double* p, const double* q, double* out);
+
 /* Copy the whole state of `src` into `dst`: every character's live KV,
  * positions, recurrent states, live lengths and cursors (§4.2: task-specific
  * continuations branch from a maintained root).  Both contexts must have the
@@ -325,7 +429,7 @@ kvm_status kvm_fork(kvm_ctx* dst, const kvm_ctx* src, void* stream);
  * reads); launches beyond it are neither timed nor counted here
  * (kvm_launch_count counts every launch). */
 enum { KVM_K_COMPACT = 0, KVM_K_ROPE_APPEND = 1, KVM_K_ATTENTION = 2, KVM_K_ATTN_COMBINE = 3,
-       KVM_K_GDN = 4, KVM_K_GATHER = 5, KVM_K_GDN_PREP = 6, KVM_K_COUNT = 7 };
+       KVM_K_GDN = 4, KVM_K_GATHER = 5, KVM_K_GDN_PREP = 6, KVM_K_GDN_CONV = 7, KVM_K_COUNT = 8 };
 kvm_status kvm_profile_enable(kvm_ctx* ctx, int32_t enable);
 kvm_status kvm_profile_read(kvm_ctx* ctx, int32_t kernel, int64_t* launches, double* total_ms,
                             int32_t reset);

@@ -17,7 +17,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libkvm.so")
-SOURCES = ["kvm_api.cu", "kv_compact.cu", "tail_attn.cu", "tail_attn_tc.cu", "gdn_scan_tc.cu"]
+SOURCES = ["kvm_api.cu", "kv_compact.cu", "tail_attn.cu", "tail_attn_tc.cu", "gdn_scan_tc.cu", "attn_probe.cu", "gdn_conv.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-cudart", "static"]

@@ -70,6 +70,8 @@ struct kvm_ctx {
     int Hq = 0, Hkv = 0, D = 0, R = 0, g = 0;
     double theta = 0;
     int H = 0, dk = 0, dv = 0;
+    int conv = 0;                         // short-convolution width of the delta-rule layers (0 or 4)
+    int conv_ch = 0;                      // its channels, H (2 d_k + d_v)
     // population
     int B = 0;
     std::vector<int> cap, cap_off;
@@ -85,6 +87,24 @@ struct kvm_ctx {
     float* S = nullptr;
     // workspace
     __nv_bfloat16* q_rot = nullptr;
+    // per-token positions (tail placement variants) and re-rotation targets:
+    // host values go through a pinned staging buffer, guarded by ev_pos
+    int32_t* tail_pos_dev = nullptr;      // [max_tail]
+    int32_t* reloc_pos_dev = nullptr;     // [max capacity]
+    int32_t* pos_host = nullptr;          // pinned [max(max_tail, max capacity)]
+    cudaEvent_t ev_pos = nullptr;
+    int max_cap = 0;
+    // attention-probe workspace: rotated probe queries, per-tile and per-row softmax partials
+    // short convolution: weights [n_gdn][C][4] fp32; state, two buffers per
+    // layer [2][n_gdn][B][3][C] bf16 (a round reads one, writes the other,
+    // conv_par[layer] tells which is current); outputs [max_tail][H][...] bf16
+    float* conv_w = nullptr;
+    __nv_bfloat16* conv_state = nullptr;
+    std::vector<int> conv_par;
+    __nv_bfloat16* conv_y = nullptr;
+    float* probe_q = nullptr;
+    float* probe_part = nullptr;
+    float* probe_rows = nullptr;
     float* part_o = nullptr;
     float* part_ml = nullptr;
     int32_t* tickets = nullptr;
@@ -135,6 +155,16 @@ void free_all(kvm_ctx* c) {
                     c->flags, c->err, c->stage, c->gdn_work, c->diag};
     for (void* p : ptrs)
         if (p) cudaFree(p);
+    if (c->tail_pos_dev) cudaFree(c->tail_pos_dev);
+    if (c->probe_q) cudaFree(c->probe_q);
+    if (c->conv_w) cudaFree(c->conv_w);
+    if (c->conv_state) cudaFree(c->conv_state);
+    if (c->conv_y) cudaFree(c->conv_y);
+    if (c->probe_part) cudaFree(c->probe_part);
+    if (c->probe_rows) cudaFree(c->probe_rows);
+    if (c->reloc_pos_dev) cudaFree(c->reloc_pos_dev);
+    if (c->pos_host) cudaFreeHost(c->pos_host);
+    if (c->ev_pos) cudaEventDestroy(c->ev_pos);
     for (cudaEvent_t e : c->ev_in) if (e) cudaEventDestroy(e);
     for (cudaEvent_t e : c->ev_done) if (e) cudaEventDestroy(e);
     if (c->ev_start) cudaEventDestroy(c->ev_start);
@@ -183,6 +213,33 @@ int prof_begin(kvm_ctx* c, int kind, cudaStream_t s) {
 
 void prof_end(kvm_ctx* c, int slot, cudaStream_t s) {
     if (slot >= 0) cudaEventRecord(c->ev[2 * slot + 1], s);
+}
+
+// Copy n host positions into the device buffer dev on stream s through the
+// context's pinned staging buffer (the previous staging copy must have left
+// it first, which ev_pos tracks).
+kvm_status stage_positions(kvm_ctx* c, const int32_t* host, int n, int32_t* dev, cudaStream_t s) {
+    if (n <= 0) return KVM_OK;
+    CUDA_TRY(cudaEventSynchronize(c->ev_pos));
+    std::memcpy(c->pos_host, host, sizeof(int32_t) * (size_t)n);
+    CUDA_TRY(cudaMemcpyAsync(dev, c->pos_host, sizeof(int32_t) * (size_t)n, cudaMemcpyHostToDevice, s));
+    CUDA_TRY(cudaEventRecord(c->ev_pos, s));
+    return KVM_OK;
+}
+
+// Per-token positions, if given, must be non-negative (they are int32, so
+// no id passes 2^31 - 1); without them the cursor must leave room for M ids.
+kvm_status check_positions(const kvm_ctx* c, const int32_t* tail_cu, const int32_t* tail_pos) {
+    for (int b = 0; b < c->B; ++b) {
+        const int m = tail_cu[b + 1] - tail_cu[b];
+        if (tail_pos) {
+            for (int i = tail_cu[b]; i < tail_cu[b + 1]; ++i)
+                if (tail_pos[i] < 0) return fail(KVM_E_INVAL, "character %d: tail position %d is negative", b, i);
+        } else if (c->cursor[b] + m > INT32_MAX) {
+            return fail(KVM_E_CAPACITY, "character %d: position ids overflow", b);
+        }
+    }
+    return KVM_OK;
 }
 
 // Validate one round's spans and build the per-character segment tables.
@@ -356,6 +413,12 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         if (c->H <= 0) { delete c; return fail(KVM_E_INVAL, "n_gdn_heads must be positive"); }
         if (c->dk != 64 && c->dk != 128) { delete c; return fail(KVM_E_UNSUPPORTED, "d_k must be 64 or 128"); }
         if (c->dv <= 0 || c->dv % 32 || c->dv > 128) { delete c; return fail(KVM_E_UNSUPPORTED, "d_v must be a multiple of 32, <= 128"); }
+        if (m->conv_kernel != 0 && m->conv_kernel != 4) { delete c; return fail(KVM_E_UNSUPPORTED, "conv_kernel must be 0 or 4"); }
+        c->conv = m->conv_kernel;
+        c->conv_ch = c->H * (2 * c->dk + c->dv);
+    } else if (m->conv_kernel != 0 && m->conv_kernel != 4) {
+        delete c;
+        return fail(KVM_E_UNSUPPORTED, "conv_kernel must be 0 or 4");
     }
     c->B = n_chars;
     c->max_tail = max_tail_tokens;
@@ -392,6 +455,26 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
     if (e == cudaSuccess) e = alloc_zero(&c->pos, c->n_attn ? (size_t)c->T_cap : 0);
     if (e == cudaSuccess) e = alloc_zero(&c->S, (size_t)c->n_gdn * n_chars * c->H * c->dv * c->dk);
     if (e == cudaSuccess) e = alloc_zero(&c->q_rot, c->n_attn ? (size_t)max_tail_tokens * c->Hq * c->D : 0);
+    for (int b = 0; b < n_chars; ++b) c->max_cap = std::max(c->max_cap, c->cap[b]);
+    if (e == cudaSuccess) e = alloc_zero(&c->tail_pos_dev, c->n_attn ? (size_t)max_tail_tokens : 0);
+    if (e == cudaSuccess) e = alloc_zero(&c->reloc_pos_dev, c->n_attn ? (size_t)c->max_cap : 0);
+    if (e == cudaSuccess && c->n_attn)
+        e = cudaHostAlloc(reinterpret_cast<void**>(&c->pos_host),
+                          sizeof(int32_t) * std::max(max_tail_tokens, c->max_cap), cudaHostAllocDefault);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_pos, cudaEventDisableTiming);
+    if (c->conv) {
+        c->conv_par.assign(c->n_gdn, 0);
+        if (e == cudaSuccess) e = alloc_zero(&c->conv_w, (size_t)c->n_gdn * c->conv_ch * 4);
+        if (e == cudaSuccess) e = alloc_zero(&c->conv_state, (size_t)2 * c->n_gdn * n_chars * 3 * c->conv_ch);
+        if (e == cudaSuccess) e = alloc_zero(&c->conv_y, (size_t)max_tail_tokens * c->conv_ch);
+    }
+    if (c->n_attn) {
+        const size_t rows = (size_t)kProbeMaxQueries * c->Hq;
+        const size_t tiles = ((size_t)c->max_cap + kProbeKeys - 1) / kProbeKeys;
+        if (e == cudaSuccess) e = alloc_zero(&c->probe_q, rows * c->D);
+        if (e == cudaSuccess) e = alloc_zero(&c->probe_part, tiles * rows * 2);
+        if (e == cudaSuccess) e = alloc_zero(&c->probe_rows, rows * 2);
+    }
     const size_t part_slots = c->n_attn ? 2 * (size_t)attention_grid_cap(c->num_sms, c->D) : 0;
     if (e == cudaSuccess) e = alloc_zero(&c->part_o, part_slots * kAttnRows * c->D);
     if (e == cudaSuccess) e = alloc_zero(&c->part_ml, part_slots * kAttnRows * 2);
@@ -566,6 +649,52 @@ extern "C" kvm_status kvm_get_state(kvm_ctx* c, int32_t layer, float* S, void* s
     return KVM_OK;
 }
 
+namespace {
+kvm_status check_conv_layer(const kvm_ctx* c, int layer) {
+    kvm_status st = check_layer(c, layer, KVM_LAYER_GDN);
+    if (st) return st;
+    if (!c->conv) return fail(KVM_E_INVAL, "the context has no short convolution (conv_kernel = 0)");
+    return KVM_OK;
+}
+// Current conv state buffer of a delta-rule layer ([B][3][C] bf16).
+__nv_bfloat16* conv_state_of(kvm_ctx* c, int g, int which) {
+    return c->conv_state + ((size_t)which * c->n_gdn + g) * c->B * 3 * c->conv_ch;
+}
+}  // namespace
+
+extern "C" kvm_status kvm_set_conv_weights(kvm_ctx* c, int32_t layer, const float* w, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    kvm_status st = check_conv_layer(c, layer);
+    if (st) return st;
+    if (!w) return fail(KVM_E_INVAL, "NULL weights");
+    const size_t n = (size_t)c->conv_ch * 4;
+    CUDA_TRY(cudaMemcpyAsync(c->conv_w + (size_t)c->gdn_idx[layer] * n, w, n * 4, cudaMemcpyDeviceToDevice,
+                             (cudaStream_t)stream));
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_get_conv_state(kvm_ctx* c, int32_t layer, void* out, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    kvm_status st = check_conv_layer(c, layer);
+    if (st) return st;
+    if (!out) return fail(KVM_E_INVAL, "NULL output");
+    const int g = c->gdn_idx[layer];
+    CUDA_TRY(cudaMemcpyAsync(out, conv_state_of(c, g, c->conv_par[g]), (size_t)c->B * 3 * c->conv_ch * 2,
+                             cudaMemcpyDeviceToDevice, (cudaStream_t)stream));
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_set_conv_state(kvm_ctx* c, int32_t layer, const void* in, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    kvm_status st = check_conv_layer(c, layer);
+    if (st) return st;
+    if (!in) return fail(KVM_E_INVAL, "NULL state");
+    const int g = c->gdn_idx[layer];
+    CUDA_TRY(cudaMemcpyAsync(conv_state_of(c, g, c->conv_par[g]), in, (size_t)c->B * 3 * c->conv_ch * 2,
+                             cudaMemcpyDeviceToDevice, (cudaStream_t)stream));
+    return KVM_OK;
+}
+
 extern "C" kvm_status kvm_get_live(kvm_ctx* c, int32_t b, int32_t* live, int64_t* cursor) {
     if (!c) return fail(KVM_E_INVAL, "NULL context");
     if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
@@ -627,18 +756,39 @@ extern "C" kvm_status kvm_plan_attention(int32_t n_chars, const int32_t* live, c
 }
 
 namespace {
-// Position ranges -> live-index spans over the sorted live positions P[live].
+// Position ranges -> live-index spans over the live positions P[live].
+// Positions are in live order; they increase unless per-token positions or
+// re-rotation placed entries out of order.  Each range must cover at least
+// one live entry, and the entries it covers must be one contiguous run of
+// live indices (always true when the positions increase).
 kvm_status spans_from_positions(const int32_t* P, int live, int32_t n, const int64_t* pb, const int64_t* pe,
                                 int32_t* sb, int32_t* se) {
     if (n < 0) return fail(KVM_E_INVAL, "negative count");
     if (n > 0 && (!pb || !pe || !sb || !se)) return fail(KVM_E_INVAL, "NULL argument");
+    bool increasing = true;
+    for (int i = 1; i < live && increasing; ++i) increasing = P[i] > P[i - 1];
     int64_t prev_end = INT64_MIN;
     for (int i = 0; i < n; ++i) {
         if (pb[i] >= pe[i]) return fail(KVM_E_SPAN, "position range %d is empty", i);
         if (pb[i] < prev_end) return fail(KVM_E_SPAN, "position range %d overlaps or precedes the previous one", i);
         prev_end = pe[i];
-        const int lo = (int)(std::lower_bound(P, P + live, pb[i]) - P);
-        const int hi = (int)(std::lower_bound(P, P + live, pe[i]) - P);
+        int lo, hi;
+        if (increasing) {
+            lo = (int)(std::lower_bound(P, P + live, pb[i]) - P);
+            hi = (int)(std::lower_bound(P, P + live, pe[i]) - P);
+        } else {
+            lo = live;
+            hi = -1;
+            int count = 0;
+            for (int j = 0; j < live; ++j)
+                if (P[j] >= pb[i] && P[j] < pe[i]) {
+                    lo = std::min(lo, j);
+                    hi = std::max(hi, j + 1);
+                    ++count;
+                }
+            if (count > 0 && count != hi - lo)
+                return fail(KVM_E_SPAN, "position range %d covers live entries that are not one contiguous run", i);
+        }
         if (hi <= lo) return fail(KVM_E_SPAN, "position range %d covers no live entry", i);
         sb[i] = lo;
         se[i] = hi;
@@ -660,8 +810,8 @@ extern "C" kvm_status kvm_plan_spans_from_positions(int32_t live, const int32_t*
                                                     int32_t* span_begin, int32_t* span_end) {
     if (live < 0) return fail(KVM_E_INVAL, "negative live length");
     if (live > 0 && !positions) return fail(KVM_E_INVAL, "positions is NULL");
-    for (int i = 1; i < live; ++i)
-        if (positions[i] <= positions[i - 1]) return fail(KVM_E_INVAL, "positions must be strictly increasing");
+    for (int i = 0; i < live; ++i)
+        if (positions[i] < 0) return fail(KVM_E_INVAL, "positions must be non-negative");
     return spans_from_positions(positions, live, n, pos_begin, pos_end, span_begin, span_end);
 }
 
@@ -784,8 +934,12 @@ kvm_status do_compact(kvm_ctx* c, const int32_t* span_cu, const int32_t* sbeg, c
     return KVM_OK;
 }
 
+// tail_pos_dev: device positions of the tail tokens (already staged), or
+// null for the true tail p_b + i; tail_pos_host: the same values on the host
+// for validation (null when tail_pos_dev is null).
 kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, const void* k_new,
-                        const void* v_new, void* out, cudaStream_t s) {
+                        const void* v_new, void* out, cudaStream_t s, const int32_t* tail_pos_dev = nullptr,
+                        const int32_t* tail_pos_host = nullptr) {
     kvm_status st = check_layer(c, layer, KVM_LAYER_ATTN);
     if (st) return st;
     int total = 0;
@@ -796,8 +950,9 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
         if (c->live[b] + m > c->cap[b])
             return fail(KVM_E_CAPACITY, "character %d: live %d + tail %d exceeds capacity %d", b, c->live[b], m,
                         c->cap[b]);
-        if (c->cursor[b] + m > INT32_MAX) return fail(KVM_E_CAPACITY, "character %d: position ids overflow", b);
     }
+    st = check_positions(c, tail_cu, tail_pos_host);
+    if (st) return st;
     if (total == 0) return KVM_OK;
     if (!q || !k_new || !v_new || !out) return fail(KVM_E_INVAL, "NULL tensor");
 
@@ -820,6 +975,7 @@ kvm_status do_attention(kvm_ctx* c, int layer, const int32_t* tail_cu, const voi
     p.V = c->V + (size_t)a * c->Hkv * c->T_cap * c->D;
     p.pos = c->pos;
     p.out = static_cast<__nv_bfloat16*>(out);
+    p.tail_pos = tail_pos_dev;
     p.part_o = c->part_o;
     p.part_ml = c->part_ml;
     p.err = c->err;
@@ -892,6 +1048,31 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
     p.q = static_cast<const __nv_bfloat16*>(q);
     p.k = static_cast<const __nv_bfloat16*>(k);
     p.v = static_cast<const __nv_bfloat16*>(v);
+    if (c->conv) {
+        // short convolution + SiLU (+ k normalisation) from the carried conv
+        // state; the delta rule then reads the convolved q, k, v
+        thread_local static ConvParams cp;
+        std::memset(&cp, 0, sizeof cp);
+        const int g = c->gdn_idx[layer];
+        cp.n_chars = c->B;
+        cp.H = c->H; cp.dk = c->dk; cp.dv = c->dv; cp.channels = c->conv_ch;
+        cp.total = total;
+        for (int b = 0; b <= c->B; ++b) cp.tail_cu[b] = tail_cu[b];
+        cp.xq = p.q; cp.xk = p.k; cp.xv = p.v;
+        cp.w = c->conv_w + (size_t)g * c->conv_ch * 4;
+        cp.state_in = conv_state_of(c, g, c->conv_par[g]);
+        cp.state_out = conv_state_of(c, g, c->conv_par[g] ^ 1);
+        cp.yq = c->conv_y;
+        cp.yk = cp.yq + (size_t)total * c->H * c->dk;
+        cp.yv = cp.yk + (size_t)total * c->H * c->dk;
+        cp.err = c->err;
+        const int ps = prof_begin(c, KVM_K_GDN_CONV, s);
+        launch_gdn_conv(cp, s);
+        prof_end(c, ps, s);
+        LAUNCH_CHECK(c);
+        c->conv_par[g] ^= 1;
+        p.q = cp.yq; p.k = cp.yk; p.v = cp.yv;
+    }
     p.alpha = alpha;
     p.beta = beta;
     p.out = static_cast<__nv_bfloat16*>(out);
@@ -923,12 +1104,25 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
     return KVM_OK;
 }
 
-void do_advance(kvm_ctx* c, const int32_t* tail_cu) {
+// End of a round: live lengths grow by M; the host position mirror gets the
+// tail's positions; the cursor moves to p + M (true tail) or, with per-token
+// positions, past the largest position used (it never moves back).
+void do_advance(kvm_ctx* c, const int32_t* tail_cu, const int32_t* tail_pos = nullptr) {
     for (int b = 0; b < c->B; ++b) {
         const int m = tail_cu[b + 1] - tail_cu[b];
-        for (int i = 0; i < m; ++i) c->hpos[b].push_back((int32_t)(c->cursor[b] + i));
+        if (tail_pos) {
+            int64_t top = c->cursor[b];
+            for (int i = 0; i < m; ++i) {
+                const int32_t x = tail_pos[tail_cu[b] + i];
+                c->hpos[b].push_back(x);
+                top = std::max<int64_t>(top, (int64_t)x + 1);
+            }
+            c->cursor[b] = top;
+        } else {
+            for (int i = 0; i < m; ++i) c->hpos[b].push_back((int32_t)(c->cursor[b] + i));
+            c->cursor[b] += m;
+        }
         c->live[b] += m;
-        c->cursor[b] += m;
     }
 }
 
@@ -946,6 +1140,133 @@ extern "C" kvm_status kvm_tail_attn_prefill(kvm_ctx* c, int32_t layer, const int
     return do_attention(c, layer, tail_cu, q, k_new, v_new, out, (cudaStream_t)stream);
 }
 
+extern "C" kvm_status kvm_tail_attn_prefill_at(kvm_ctx* c, int32_t layer, const int32_t* tail_cu,
+                                               const int32_t* tail_pos, const void* q, const void* k_new,
+                                               const void* v_new, void* out, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (!tail_pos) return do_attention(c, layer, tail_cu, q, k_new, v_new, out, (cudaStream_t)stream);
+    kvm_status st = check_layer(c, layer, KVM_LAYER_ATTN);
+    if (st) return st;
+    int total = 0;
+    st = check_tail_cu(c, tail_cu, &total);
+    if (st) return st;
+    st = check_positions(c, tail_cu, tail_pos);
+    if (st) return st;
+    for (int b = 0; b < c->B; ++b)
+        if (c->live[b] + tail_cu[b + 1] - tail_cu[b] > c->cap[b])
+            return fail(KVM_E_CAPACITY, "character %d: live + tail exceeds capacity", b);
+    if (total > 0 && (!q || !k_new || !v_new || !out)) return fail(KVM_E_INVAL, "NULL tensor");
+    st = stage_positions(c, tail_pos, total, c->tail_pos_dev, (cudaStream_t)stream);
+    if (st) return st;
+    return do_attention(c, layer, tail_cu, q, k_new, v_new, out, (cudaStream_t)stream, c->tail_pos_dev, tail_pos);
+}
+
+extern "C" kvm_status kvm_rerotate_keys(kvm_ctx* c, int32_t b, int32_t live_begin, int32_t live_end,
+                                        const int32_t* new_pos, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (c->n_attn == 0) return fail(KVM_E_INVAL, "the model has no attention layer");
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    if (!(0 <= live_begin && live_begin <= live_end && live_end <= c->live[b]))
+        return fail(KVM_E_SPAN, "range [%d,%d) outside the live entries [0,%d)", live_begin, live_end, c->live[b]);
+    const int n = live_end - live_begin;
+    if (n == 0) return KVM_OK;
+    if (!new_pos) return fail(KVM_E_INVAL, "new_pos is NULL");
+    int64_t top = c->cursor[b];
+    for (int i = 0; i < n; ++i) {
+        if (new_pos[i] < 0) return fail(KVM_E_INVAL, "new position %d is negative", i);
+        top = std::max<int64_t>(top, (int64_t)new_pos[i] + 1);
+    }
+    cudaStream_t s = (cudaStream_t)stream;
+    kvm_status st = stage_positions(c, new_pos, n, c->reloc_pos_dev, s);
+    if (st) return st;
+    RerotateParams p;
+    std::memset(&p, 0, sizeof p);
+    p.n = n;
+    p.n_attn = c->n_attn;
+    p.Hkv = c->Hkv;
+    p.D = c->D;
+    p.R = c->R;
+    p.slot0 = (int64_t)c->cap_off[b] + live_begin;
+    p.slab_rows = c->T_cap;
+    p.K = c->K;
+    p.pos = c->pos;
+    p.new_pos = c->reloc_pos_dev;
+    p.err = c->err;
+    for (int d = 0; d < c->R / 2; ++d) p.inv_freq[d] = c->inv_freq[d];
+    ++c->launches;
+    launch_rerotate(p, s);
+    LAUNCH_CHECK(c);
+    for (int i = 0; i < n; ++i) c->hpos[b][live_begin + i] = new_pos[i];
+    c->cursor[b] = top;
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_attn_probe(kvm_ctx* c, int32_t layer, int32_t b, int32_t n_q, const void* q,
+                                     float* probs_out, const int32_t* group_of, int32_t n_groups,
+                                     float* group_mass_out, void* stream) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    kvm_status st = check_layer(c, layer, KVM_LAYER_ATTN);
+    if (st) return st;
+    if (b < 0 || b >= c->B) return fail(KVM_E_INVAL, "character %d out of range", b);
+    const int L = c->live[b];
+    if (n_q < 1 || n_q > kProbeMaxQueries || n_q > L)
+        return fail(KVM_E_INVAL, "n_q must be in [1, min(%d, live = %d)]", kProbeMaxQueries, L);
+    if (!q || !probs_out) return fail(KVM_E_INVAL, "NULL q or probs_out");
+    if (group_of && (n_groups < 1 || !group_mass_out))
+        return fail(KVM_E_INVAL, "group_of needs n_groups >= 1 and group_mass_out");
+    cudaStream_t s = (cudaStream_t)stream;
+    ProbeParams p;
+    std::memset(&p, 0, sizeof p);
+    p.L = L;
+    p.n_q = n_q;
+    p.Hq = c->Hq; p.Hkv = c->Hkv; p.D = c->D; p.R = c->R; p.g = c->g;
+    p.n_groups = group_of ? n_groups : 0;
+    p.scale = (float)(1.0 / std::sqrt((double)c->D));
+    p.slab_rows = c->T_cap;
+    p.slot0 = c->cap_off[b];
+    p.q = static_cast<const __nv_bfloat16*>(q);
+    p.q_rot = c->probe_q;
+    p.K = c->K + (size_t)c->attn_idx[layer] * c->Hkv * c->T_cap * c->D;
+    p.pos = c->pos;
+    p.part = c->probe_part;
+    p.row_ms = c->probe_rows;
+    p.probs = probs_out;
+    p.group_of = group_of;
+    p.group_mass = group_mass_out;
+    p.err = c->err;
+    for (int d = 0; d < c->R / 2; ++d) p.inv_freq[d] = c->inv_freq[d];
+    if (group_of) CUDA_TRY(cudaMemsetAsync(group_mass_out, 0, sizeof(float) * (size_t)n_groups, s));
+    c->launches += 4;
+    launch_attn_probe(p, s);
+    LAUNCH_CHECK(c);
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_effective_group_count(int32_t n_groups, const double* mass, double* out) {
+    if (n_groups < 1 || !mass || !out) return fail(KVM_E_INVAL, "need n_groups >= 1, mass and out");
+    double tot = 0.0;
+    for (int i = 0; i < n_groups; ++i) {
+        if (!(mass[i] >= 0.0)) return fail(KVM_E_INVAL, "group mass %d is negative or NaN", i);
+        tot += mass[i];
+    }
+    if (!(tot > 0.0)) return fail(KVM_E_INVAL, "the groups carry no mass");
+    double h = 0.0;                                  // entropy of the normalised group probabilities
+    for (int i = 0; i < n_groups; ++i) {
+        const double a = mass[i] / tot;
+        if (a > 0.0) h -= a * std::log(a);
+    }
+    *out = std::exp(h);
+    return KVM_OK;
+}
+
+extern "C" kvm_status kvm_total_variation(int32_t n, const double* p, const double* q, double* out) {
+    if (n < 0 || (n > 0 && (!p || !q)) || !out) return fail(KVM_E_INVAL, "need n >= 0, p, q and out");
+    double d = 0.0;
+    for (int i = 0; i < n; ++i) d += std::fabs(p[i] - q[i]);
+    *out = 0.5 * d;
+    return KVM_OK;
+}
+
 extern "C" kvm_status kvm_gdn_chunk_scan_from_state(kvm_ctx* c, int32_t layer, const int32_t* tail_cu,
                                                     const void* q, const void* k, const void* v,
                                                     const float* alpha, const float* beta, void* out,
@@ -954,7 +1275,7 @@ extern "C" kvm_status kvm_gdn_chunk_scan_from_state(kvm_ctx* c, int32_t layer, c
     return do_gdn(c, layer, tail_cu, q, k, v, alpha, beta, out, (cudaStream_t)stream);
 }
 
-extern "C" kvm_status kvm_advance(kvm_ctx* c, const int32_t* tail_cu) {
+extern "C" kvm_status kvm_advance_at(kvm_ctx* c, const int32_t* tail_cu, const int32_t* tail_pos) {
     if (!c) return fail(KVM_E_INVAL, "NULL context");
     int total = 0;
     kvm_status st = check_tail_cu(c, tail_cu, &total);
@@ -962,9 +1283,13 @@ extern "C" kvm_status kvm_advance(kvm_ctx* c, const int32_t* tail_cu) {
     for (int b = 0; b < c->B; ++b)
         if (c->live[b] + tail_cu[b + 1] - tail_cu[b] > c->cap[b])
             return fail(KVM_E_CAPACITY, "character %d would exceed its capacity", b);
-    do_advance(c, tail_cu);
+    st = check_positions(c, tail_cu, tail_pos);
+    if (st) return st;
+    do_advance(c, tail_cu, tail_pos);
     return KVM_OK;
 }
+
+extern "C" kvm_status kvm_advance(kvm_ctx* c, const int32_t* tail_cu) { return kvm_advance_at(c, tail_cu, nullptr); }
 
 extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* stream) {
     if (!c || !r) return fail(KVM_E_INVAL, "NULL argument");
@@ -983,14 +1308,25 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
             if (pl.L_new[b] + m > c->cap[b])
                 return fail(KVM_E_CAPACITY, "character %d: live %d + tail %d exceeds capacity %d", b, pl.L_new[b],
                             m, c->cap[b]);
-            if (c->cursor[b] + m > INT32_MAX) return fail(KVM_E_CAPACITY, "character %d: position ids overflow", b);
         }
+        st = check_positions(c, r->tail_cu, r->tail_pos);
+        if (st) return st;
         for (int l = 0; l < c->n_layers; ++l) {
             if (total > 0 && (!r->q[l] || !r->k[l] || !r->v[l] || !r->out[l]))
                 return fail(KVM_E_INVAL, "layer %d has a NULL tensor", l);
             if (c->kind[l] == KVM_LAYER_GDN && total > 0 && (!r->alpha || !r->beta || !r->alpha[l] || !r->beta[l]))
                 return fail(KVM_E_INVAL, "layer %d has NULL gates", l);
         }
+    }
+    // maintenance delimiters: tail-index spans [s, e) of each character's
+    // tail, checked like removal spans against the tail length
+    std::vector<int> tail_len(c->B);
+    for (int b = 0; b < c->B; ++b) tail_len[b] = r->tail_cu[b + 1] - r->tail_cu[b];
+    SpanPlan delim_plan;
+    const bool has_delim = r->delim_cu && r->delim_cu[c->B] > 0;
+    if (has_delim) {
+        st = plan_spans_for(c->B, tail_len.data(), r->delim_cu, r->delim_begin, r->delim_end, delim_plan);
+        if (st) return st;
     }
     const bool host_io = r->io_on_host && total > 0;
     auto sizes = [&](int l, size_t n[6]) {
@@ -1072,6 +1408,11 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
         if (side) CUDA_TRY(cudaEventRecord(c->ev_compacted, cs));
         apply_plan(c, pl, r->span_cu, r->span_begin, r->span_end);
     }
+    const bool with_pos = r->tail_pos && total > 0 && c->n_attn > 0;
+    if (with_pos) {
+        st = stage_positions(c, r->tail_pos, total, c->tail_pos_dev, s);
+        if (st) return st;
+    }
     const int join_at = first_attn >= 2 ? first_attn - 1 : first_attn;
     bool joined = !side;
     auto join = [&]() -> cudaError_t {
@@ -1096,7 +1437,8 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
             }
             out = c->stage + c->stage_out_off[l];
         }
-        st = attn ? do_attention(c, l, r->tail_cu, q, k, v, out, s)
+        st = attn ? do_attention(c, l, r->tail_cu, q, k, v, out, s, with_pos ? c->tail_pos_dev : nullptr,
+                                 with_pos ? r->tail_pos : nullptr)
                   : do_gdn(c, l, r->tail_cu, q, k, v, al, be, out, s);
         if (st) {
             join();                                   // s still covers the compaction
@@ -1117,7 +1459,27 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
         CUDA_TRY(cudaEventRecord(c->ev_copies, c->copy_stream));
         CUDA_TRY(cudaStreamWaitEvent(s, c->ev_copies, 0));
     }
-    do_advance(c, r->tail_cu);
+    std::vector<int> L_round(c->live);              // L'_b: where each tail was appended
+    do_advance(c, r->tail_cu, r->tail_pos);
+    if (has_delim) {
+        // the delimiters' direct KV leave every attention layer; their
+        // effect on the recurrent states and on later tail tokens stays
+        std::vector<int32_t> cu(c->B + 1), sb, se;
+        for (int b = 0; b < c->B; ++b) {
+            cu[b] = (int32_t)sb.size();
+            for (int k = r->delim_cu[b]; k < r->delim_cu[b + 1]; ++k) {
+                sb.push_back(L_round[b] + r->delim_begin[k]);
+                se.push_back(L_round[b] + r->delim_end[k]);
+            }
+        }
+        cu[c->B] = (int32_t)sb.size();
+        SpanPlan pl;
+        st = plan_spans(c, cu.data(), sb.data(), se.data(), pl);
+        if (st) return st;                            // cannot happen: checked against the tails above
+        st = launch_compaction(c, pl, s, 0, c->n_attn, true);
+        if (st) return st;
+        apply_plan(c, pl, cu.data(), sb.data(), se.data());
+    }
     return KVM_OK;
 }
 
@@ -1151,7 +1513,7 @@ extern "C" kvm_status kvm_fork(kvm_ctx* dst, const kvm_ctx* src, void* stream) {
     if (dst == src) return KVM_OK;
     if (dst->kind != src->kind || dst->Hq != src->Hq || dst->Hkv != src->Hkv || dst->D != src->D ||
         dst->R != src->R || dst->theta != src->theta || dst->H != src->H || dst->dk != src->dk ||
-        dst->dv != src->dv || dst->B != src->B || dst->cap != src->cap)
+        dst->dv != src->dv || dst->B != src->B || dst->cap != src->cap || dst->conv != src->conv)
         return fail(KVM_E_INVAL, "contexts differ in model shape, population or capacity");
     cudaStream_t s = (cudaStream_t)stream;
     const size_t kv = (size_t)src->n_attn * src->Hkv * src->T_cap * src->D * sizeof(__nv_bfloat16);
@@ -1162,6 +1524,13 @@ extern "C" kvm_status kvm_fork(kvm_ctx* dst, const kvm_ctx* src, void* stream) {
     }
     const size_t sn = (size_t)src->n_gdn * src->B * src->H * src->dv * src->dk * sizeof(float);
     if (sn) CUDA_TRY(cudaMemcpyAsync(dst->S, src->S, sn, cudaMemcpyDeviceToDevice, s));
+    if (src->conv) {
+        const size_t cs = (size_t)2 * src->n_gdn * src->B * 3 * src->conv_ch * 2;
+        CUDA_TRY(cudaMemcpyAsync(dst->conv_state, src->conv_state, cs, cudaMemcpyDeviceToDevice, s));
+        CUDA_TRY(cudaMemcpyAsync(dst->conv_w, src->conv_w, (size_t)src->n_gdn * src->conv_ch * 4 * 4,
+                                 cudaMemcpyDeviceToDevice, s));
+        dst->conv_par = src->conv_par;
+    }
     dst->live = src->live;
     dst->cursor = src->cursor;
     dst->hpos = src->hpos;

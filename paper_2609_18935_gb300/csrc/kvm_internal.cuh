@@ -142,6 +142,7 @@ struct AttnParams {
     __nv_bfloat16* V;
     int32_t* pos;                 // [slab_rows]
     __nv_bfloat16* out;           // [sum M][Hq][D]
+    const int32_t* tail_pos;      // device [sum M] position of each tail token, or null: p + i
     float* part_o;                // [2 n_ctas][D / 32][8][128][4]: partial O of a block's first / last segment
     float* part_ml;               // [2 n_ctas][128][2]: (reference max in log2 units, sum) of a partial
     int32_t* err;
@@ -155,10 +156,53 @@ struct AttnParams {
 };
 
 void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s);
+
+// Key re-rotation (tail-and-relocate, §5.2): rotate stored keys of live slots
+// [slot0, slot0 + n) in every attention layer by (new_pos - pos), then set pos.
+struct RerotateParams {
+    int32_t n;            // entries
+    int32_t n_attn, Hkv, D, R;
+    int64_t slot0;        // first slot (character offset + live index)
+    int64_t slab_rows;
+    __nv_bfloat16* K;     // all layers' K slabs [n_attn][Hkv][slab_rows][D]
+    int32_t* pos;         // [slab_rows]
+    const int32_t* new_pos;   // device [n]
+    int32_t* err;
+    double inv_freq[kMaxRotaryHalf];
+};
+void launch_rerotate(const RerotateParams& p, cudaStream_t s);
 void launch_tail_attention(const AttnParams& p, cudaStream_t s);
 void launch_attn_combine(const AttnParams& p, cudaStream_t s);
 int attention_ctas_per_sm(int head_dim);
 constexpr int kAttnRows = 128;   // query rows per attention tile
+
+// ----------------------------------------------------------------------------
+// attention-probe diagnostics (§5.3, Appendix C)
+// ----------------------------------------------------------------------------
+constexpr int kProbeMaxQueries = 16;   // probe queries per call (the paper averages the last 8)
+constexpr int kProbeKeys = 64;         // keys per probe block
+
+struct ProbeParams {
+    int32_t L;            // live entries of the character
+    int32_t n_q;          // probe queries: the last n_q live entries
+    int32_t Hq, Hkv, D, R, g;
+    int32_t n_groups;
+    float scale;          // 1 / sqrt(D)
+    int64_t slab_rows;
+    int64_t slot0;        // the character's first slot
+    const __nv_bfloat16* q;   // caller's unrotated probe queries [n_q][Hq][D]
+    float* q_rot;             // workspace [n_q][Hq][D] fp32
+    const __nv_bfloat16* K;   // this layer's K slabs [Hkv][slab_rows][D]
+    const int32_t* pos;       // [slab_rows]
+    float* part;              // workspace [ceil(L / 64)][n_q * Hq][2]: per key tile (max, sum)
+    float* row_ms;            // workspace [n_q * Hq][2]: per query row (max, sum)
+    float* probs;             // out [L]
+    const int32_t* group_of;  // [L] or null
+    float* group_mass;        // out [n_groups]
+    int32_t* err;
+    double inv_freq[kMaxRotaryHalf];
+};
+void launch_attn_probe(const ProbeParams& p, cudaStream_t s);
 
 // ----------------------------------------------------------------------------
 // gated delta rule
@@ -187,6 +231,25 @@ struct GdnParams {
     int32_t* diag;            // first expired wait: block + 1, tag, parity
     GdnChar ch[kMaxChars];
 };
+
+// Short convolution (width 4) + SiLU of a delta-rule layer's q/k/v with the
+// carried conv state; k is L2-normalised per head afterwards.
+struct ConvParams {
+    int32_t n_chars, H, dk, dv, channels;     // channels = H (2 d_k + d_v)
+    int32_t total;                            // sum M
+    int32_t tail_cu[kMaxChars + 1];
+    const __nv_bfloat16* xq;                  // caller's pre-conv inputs [sum M][H][d_k]
+    const __nv_bfloat16* xk;
+    const __nv_bfloat16* xv;                  // [sum M][H][d_v]
+    const float* w;                           // [channels][4]
+    const __nv_bfloat16* state_in;            // [n_chars][3][channels]: the last 3 inputs before the tail
+    __nv_bfloat16* state_out;                 // [n_chars][3][channels]: the last 3 inputs after it
+    __nv_bfloat16* yq;                        // outputs, laid out like the inputs
+    __nv_bfloat16* yk;
+    __nv_bfloat16* yv;
+    int32_t* err;
+};
+void launch_gdn_conv(const ConvParams& p, cudaStream_t s);
 
 // Bytes of one (chunk, head) record of the delta-rule workspace.
 int64_t gdn_record_bytes(int dk, int dv);

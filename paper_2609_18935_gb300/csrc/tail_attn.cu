@@ -7,6 +7,10 @@
 //                The angle pos * omega_d is formed and reduced modulo 2*pi in
 //                fp64 (positions far beyond the live length stay accurate),
 //                then sin/cos and the rotation run in fp32.
+//  rerotate    : tail-and-relocate (§5.2): turn stored keys from the
+//                positions they were rotated at to new positions, i.e. rotate
+//                each rotary pair by (new - old) * omega_d (rotations of a
+//                pair compose by adding angles), and relabel the positions.
 //  attn_combine : merge the partials of query tiles that the attention's
 //                persistent blocks split between them: each partial is an
 //                unnormalised accumulator with (reference max in log2 units,
@@ -55,7 +59,7 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
     const AttnChar& c = p.ch[b];
     const int i = n - c.tail_off;
     if (i < 0 || i >= c.M) { if (threadIdx.x == 0) atomicOr(p.err, kErrBounds); return; }
-    const int64_t pos = c.p + i;
+    const int64_t pos = p.tail_pos ? (int64_t)p.tail_pos[n] : c.p + i;
     const int64_t slot = c.cap_off + c.L_prev + i;
     const int half = p.R / 2;
     const int D = p.D;
@@ -242,7 +246,44 @@ __global__ void __launch_bounds__(256, 7) attn_combine_kernel(const __grid_const
     *reinterpret_cast<uint2*>(o) = make_uint2(f2_to_bf2(acc.x * inv, acc.y * inv), f2_to_bf2(acc.z * inv, acc.w * inv));
 }
 
+// One block per entry; a thread rotates 2-element pairs (d, d + R/2) of one
+// (layer, KV head) key, with the entry's angles formed once in shared memory.
+__global__ void __launch_bounds__(256) rerotate_kernel(const __grid_constant__ RerotateParams p) {
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const int j = blockIdx.x;
+    if (j >= p.n) return;
+    const int64_t slot = p.slot0 + j;
+    const int half = p.R / 2;
+    __shared__ float cs[kMaxRotaryHalf], sn[kMaxRotaryHalf];
+    const int64_t delta = (int64_t)p.new_pos[j] - (int64_t)p.pos[slot];
+    for (int d = threadIdx.x; d < half; d += blockDim.x) {
+        const double ang = (double)delta * p.inv_freq[d];
+        const double r = fma(-rint(ang * (1.0 / kTwoPi)), kTwoPi, ang);   // ang mod 2*pi, |r| <= pi
+        float sv, cv;
+        sincosf((float)r, &sv, &cv);
+        cs[d] = cv;
+        sn[d] = sv;
+    }
+    __syncthreads();
+    const int n_items = p.n_attn * p.Hkv * half;
+    for (int idx = threadIdx.x; idx < n_items; idx += blockDim.x) {
+        const int d = idx % half, kh = idx / half;          // kh = layer * Hkv + head
+        __nv_bfloat16* row = p.K + ((int64_t)kh * p.slab_rows + slot) * p.D;
+        const float x = __bfloat162float(row[d]), y = __bfloat162float(row[d + half]);
+        row[d] = __float2bfloat16_rn(x * cs[d] - y * sn[d]);
+        row[d + half] = __float2bfloat16_rn(y * cs[d] + x * sn[d]);
+    }
+    __syncthreads();                                        // every thread has read pos[slot]
+    if (threadIdx.x == 0) p.pos[slot] = p.new_pos[j];
+}
+
 }  // namespace
+
+void launch_rerotate(const RerotateParams& p, cudaStream_t s) {
+    if (p.n <= 0) return;
+    launch_pdl(rerotate_kernel, dim3(p.n), dim3(256), 0, s, p);
+}
 
 void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s) {
     if (total_tokens <= 0) return;

@@ -33,7 +33,7 @@ class ModelDesc(C.Structure):
     _fields_ = [("n_layers", C.c_int32), ("layer_kind", C.POINTER(C.c_int32)),
                 ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32), ("head_dim", C.c_int32),
                 ("rotary_dim", C.c_int32), ("rope_theta", C.c_double), ("n_gdn_heads", C.c_int32),
-                ("d_k", C.c_int32), ("d_v", C.c_int32)]
+                ("d_k", C.c_int32), ("d_v", C.c_int32), ("conv_kernel", C.c_int32)]
 
 
 class Round(C.Structure):
@@ -42,7 +42,9 @@ class Round(C.Structure):
                 ("q", C.POINTER(C.c_void_p)), ("k", C.POINTER(C.c_void_p)), ("v", C.POINTER(C.c_void_p)),
                 ("alpha", C.POINTER(C.c_void_p)), ("beta", C.POINTER(C.c_void_p)),
                 ("out", C.POINTER(C.c_void_p)), ("io_on_host", C.c_int32),
-                ("gather_out", C.c_void_p)]
+                ("gather_out", C.c_void_p), ("tail_pos", C.POINTER(C.c_int32)),
+                ("delim_cu", C.POINTER(C.c_int32)), ("delim_begin", C.POINTER(C.c_int32)),
+                ("delim_end", C.POINTER(C.c_int32))]
 
 
 # name -> (restype, argtypes)
@@ -58,6 +60,9 @@ _SIGS = {
     "kvm_get_positions": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
     "kvm_set_state": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
     "kvm_get_state": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "kvm_set_conv_weights": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "kvm_get_conv_state": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
+    "kvm_set_conv_state": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p]),
     "kvm_get_live": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int64)]),
     "kvm_spans_from_positions": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.POINTER(C.c_int64),
                                            C.POINTER(C.c_int64), C.POINTER(C.c_int32),
@@ -70,6 +75,11 @@ _SIGS = {
                                                 C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                                 C.c_void_p, C.c_void_p]),
     "kvm_advance": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32)]),
+    "kvm_tail_attn_prefill_at": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32),
+                                           C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "kvm_advance_at": (C.c_int, [C.c_void_p, C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
+    "kvm_rerotate_keys": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.POINTER(C.c_int32),
+                                    C.c_void_p]),
     "kvm_update_round": (C.c_int, [C.c_void_p, C.POINTER(Round), C.c_void_p]),
     "kvm_check": (C.c_int, [C.c_void_p, C.c_void_p]),
     "kvm_launch_count": (C.c_int64, [C.c_void_p]),
@@ -86,15 +96,20 @@ _SIGS = {
                                          C.POINTER(C.c_int32), C.c_void_p]),
     "kvm_kv_compact_noalloc_check": (C.c_int, [C.c_void_p]),
     "kvm_debug_compact_wait": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
+    "kvm_attn_probe": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                 C.c_int32, C.c_void_p, C.c_void_p]),
+    "kvm_effective_group_count": (C.c_int, [C.c_int32, C.POINTER(C.c_double), C.POINTER(C.c_double)]),
+    "kvm_total_variation": (C.c_int, [C.c_int32, C.POINTER(C.c_double), C.POINTER(C.c_double),
+                                      C.POINTER(C.c_double)]),
     "kvm_profile_enable": (C.c_int, [C.c_void_p, C.c_int32]),
     "kvm_profile_read": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64), C.POINTER(C.c_double),
                                    C.c_int32]),
 }
 
 # kernel families of kvm_profile_read
-K_COMPACT, K_ROPE_APPEND, K_ATTENTION, K_ATTN_COMBINE, K_GDN, K_GATHER, K_GDN_PREP = range(7)
+K_COMPACT, K_ROPE_APPEND, K_ATTENTION, K_ATTN_COMBINE, K_GDN, K_GATHER, K_GDN_PREP, K_GDN_CONV = range(8)
 KERNEL_NAMES = ["kv_compact", "rope_append", "tail_attention", "attn_combine", "gdn_chunk_scan", "gather_map",
-                "gdn_chunk_prep"]
+                "gdn_chunk_prep", "gdn_conv"]
 
 _lib = None
 
@@ -184,6 +199,31 @@ def kv_compact_noalloc_check(stream=None):
     _check(_lib.kvm_kv_compact_noalloc_check(_stream(stream)))
 
 
+def _f64(a) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=np.float64))
+
+
+def effective_group_count(mass) -> float:
+    """kvm_effective_group_count: exp(entropy) of the normalised group masses."""
+    load_library()
+    m = _f64(mass)
+    out = C.c_double()
+    _check(_lib.kvm_effective_group_count(len(m), m.ctypes.data_as(C.POINTER(C.c_double)), C.byref(out)))
+    return out.value
+
+
+def total_variation(p, q) -> float:
+    """kvm_total_variation: 0.5 * sum |p - q| over matched entries."""
+    load_library()
+    a, b = _f64(p), _f64(q)
+    if a.shape != b.shape:
+        raise ValueError("p and q differ in length")
+    out = C.c_double()
+    _check(_lib.kvm_total_variation(len(a), a.ctypes.data_as(C.POINTER(C.c_double)),
+                                    b.ctypes.data_as(C.POINTER(C.c_double)), C.byref(out)))
+    return out.value
+
+
 def plan_removal(live, span_cu, span_begin, span_end):
     """kvm_plan_removal: (new live lengths, first moved index) per character;
     raises KvmError with the library's status on invalid spans."""
@@ -254,12 +294,13 @@ class Context:
     """A population of character states on the current CUDA device (kvm_create)."""
 
     def __init__(self, layer_kind, n_q_heads, n_kv_heads, head_dim, rotary_dim, rope_theta,
-                 n_gdn_heads, d_k, d_v, capacity, max_tail_tokens):
+                 n_gdn_heads, d_k, d_v, capacity, max_tail_tokens, conv_kernel=0):
         lib = load_library()
         self.layer_kind = [int(x) for x in layer_kind]
         self._kinds = _i32(self.layer_kind)
         self.desc = ModelDesc(len(self.layer_kind), _p32(self._kinds), n_q_heads, n_kv_heads, head_dim,
-                              rotary_dim, float(rope_theta), n_gdn_heads, d_k, d_v)
+                              rotary_dim, float(rope_theta), n_gdn_heads, d_k, d_v, int(conv_kernel))
+        self.conv_kernel = int(conv_kernel)
         self.n_chars = len(capacity)
         self.Hq, self.Hkv, self.D, self.R = n_q_heads, n_kv_heads, head_dim, rotary_dim
         self.H, self.dk, self.dv = n_gdn_heads, d_k, d_v
@@ -314,6 +355,23 @@ class Context:
         _check(_lib.kvm_get_state(self._h, layer, _dptr(S), _stream(stream)))
         return S
 
+    def set_conv_weights(self, layer, w, stream=None):
+        """kvm_set_conv_weights: w CUDA fp32 [channels][4]."""
+        import torch
+        _check(_lib.kvm_set_conv_weights(self._h, layer, _dptr(w, torch.float32), _stream(stream)))
+
+    def get_conv_state(self, layer, stream=None):
+        """kvm_get_conv_state: CUDA bf16 [n_chars][3][channels]."""
+        import torch
+        C_ = self.H * (2 * self.dk + self.dv)
+        out = torch.empty((self.n_chars, 3, C_), dtype=torch.bfloat16, device="cuda")
+        _check(_lib.kvm_get_conv_state(self._h, layer, _dptr(out), _stream(stream)))
+        return out
+
+    def set_conv_state(self, layer, state, stream=None):
+        import torch
+        _check(_lib.kvm_set_conv_state(self._h, layer, _dptr(state, torch.bfloat16), _stream(stream)))
+
     def get_live(self, b):
         live, cur = C.c_int32(), C.c_int64()
         _check(_lib.kvm_get_live(self._h, b, C.byref(live), C.byref(cur)))
@@ -336,12 +394,27 @@ class Context:
         _check(_lib.kvm_kv_compact(self._h, _p32(cu), _p32(sb), _p32(se), _dptr(gather_out, torch.int32),
                                    _stream(stream)))
 
-    def tail_attn_prefill(self, layer, tail_cu, q, k_new, v_new, out, stream=None):
+    def tail_attn_prefill(self, layer, tail_cu, q, k_new, v_new, out, tail_pos=None, stream=None):
+        """kvm_tail_attn_prefill, or kvm_tail_attn_prefill_at when tail_pos
+        (host int32 [sum M], one position id per tail token) is given."""
         import torch
         cu = _i32(tail_cu)
         bf = torch.bfloat16
-        _check(_lib.kvm_tail_attn_prefill(self._h, layer, _p32(cu), _dptr(q, bf), _dptr(k_new, bf),
-                                          _dptr(v_new, bf), _dptr(out, bf), _stream(stream)))
+        if tail_pos is None:
+            _check(_lib.kvm_tail_attn_prefill(self._h, layer, _p32(cu), _dptr(q, bf), _dptr(k_new, bf),
+                                              _dptr(v_new, bf), _dptr(out, bf), _stream(stream)))
+        else:
+            tp = _i32(tail_pos)
+            _check(_lib.kvm_tail_attn_prefill_at(self._h, layer, _p32(cu), _p32(tp), _dptr(q, bf),
+                                                 _dptr(k_new, bf), _dptr(v_new, bf), _dptr(out, bf),
+                                                 _stream(stream)))
+
+    def rerotate_keys(self, b, live_begin, live_end, new_pos, stream=None):
+        """kvm_rerotate_keys: turn the stored keys of live entries
+        [live_begin, live_end) of character b to the position ids new_pos."""
+        np_ = _i32(new_pos)
+        _check(_lib.kvm_rerotate_keys(self._h, int(b), int(live_begin), int(live_end),
+                                      _p32(np_) if len(np_) else None, _stream(stream)))
 
     def gdn_chunk_scan_from_state(self, layer, tail_cu, q, k, v, alpha, beta, out, stream=None):
         import torch
@@ -351,16 +424,23 @@ class Context:
                                                   _dptr(v, bf), _dptr(alpha, f), _dptr(beta, f),
                                                   _dptr(out, bf), _stream(stream)))
 
-    def advance(self, tail_cu):
+    def advance(self, tail_cu, tail_pos=None):
         cu = _i32(tail_cu)
-        _check(_lib.kvm_advance(self._h, _p32(cu)))
+        if tail_pos is None:
+            _check(_lib.kvm_advance(self._h, _p32(cu)))
+        else:
+            tp = _i32(tail_pos)
+            _check(_lib.kvm_advance_at(self._h, _p32(cu), _p32(tp)))
 
     def update_round(self, span_cu, span_begin, span_end, tail_cu, inputs, outputs,
-                     io_on_host=False, gather_out=None, stream=None):
+                     io_on_host=False, gather_out=None, stream=None, tail_pos=None, delim=None):
         """One whole round (kvm_update_round).
 
         inputs[layer] = dict(q, k, v[, alpha, beta]) and outputs[layer] = tensor,
-        CUDA tensors (io_on_host=False) or pinned CPU tensors (io_on_host=True)."""
+        CUDA tensors (io_on_host=False) or pinned CPU tensors (io_on_host=True).
+        tail_pos: optional host int32 [sum M] position ids of the tail tokens.
+        delim: optional (delim_cu, delim_begin, delim_end), tail-index ranges
+        of maintenance delimiters whose KV leave the caches after the round."""
         n = len(self.layer_kind)
         arr = lambda: (C.c_void_p * n)()
         q, k, v, al, be, out = arr(), arr(), arr(), arr(), arr(), arr()
@@ -371,10 +451,27 @@ class Context:
             al[l], be[l] = ptr(x.get("alpha")), ptr(x.get("beta"))
             out[l] = ptr(outputs[l])
         cu, sb, se, tc = _i32(span_cu), _i32(span_begin), _i32(span_end), _i32(tail_cu)
+        tp = _i32(tail_pos) if tail_pos is not None else None
+        dl = tuple(_i32(x) for x in delim) if delim is not None else None
         r = Round(_p32(cu), _p32(sb), _p32(se), _p32(tc), q, k, v, al, be, out, int(bool(io_on_host)),
-                  ptr(gather_out))
-        self._keep = (cu, sb, se, tc, q, k, v, al, be, out)
+                  ptr(gather_out), _p32(tp) if tp is not None else None,
+                  *((_p32(dl[0]), _p32(dl[1]), _p32(dl[2])) if dl is not None else (None, None, None)))
+        self._keep = (cu, sb, se, tc, q, k, v, al, be, out, tp, dl)
         _check(_lib.kvm_update_round(self._h, C.byref(r), _stream(stream)))
+
+    def attn_probe(self, layer, b, q, group_of=None, n_groups=0, stream=None):
+        """kvm_attn_probe: the probe distribution over character b's live
+        entries (CUDA fp32 [live]) for the unrotated queries q (CUDA bf16
+        [n_q][Hq][D]) of its last n_q live entries, and the per-group mass
+        (CUDA fp32 [n_groups]) when group_of (CUDA int32 [live]) is given."""
+        import torch
+        live, _ = self.get_live(b)
+        probs = torch.empty(live, dtype=torch.float32, device="cuda")
+        mass = torch.empty(max(1, n_groups), dtype=torch.float32, device="cuda") if group_of is not None else None
+        _check(_lib.kvm_attn_probe(self._h, int(layer), int(b), int(q.shape[0]), _dptr(q, torch.bfloat16),
+                                   _dptr(probs), _dptr(group_of, torch.int32), int(n_groups), _dptr(mass),
+                                   _stream(stream)))
+        return probs, mass
 
     def check(self, stream=None):
         _check(_lib.kvm_check(self._h, _stream(stream)))

@@ -67,7 +67,9 @@ class Pair:
                     self.ctx.set_kv(l, b, to_torch_bf16(K).cuda(), to_torch_bf16(V).cuda())
                 caches[l] = O.AttnCache(O.bf16_to_f64(K), O.bf16_to_f64(V), pos.astype(np.int64))
             for l in s.gdn_layers:
-                if prefix == "refill" and n > 0:
+                if prefix == "empty":
+                    S32 = np.zeros((s.n_gdn_heads, s.d_v, s.d_k), np.float32)
+                elif prefix == "refill" and n > 0:
                     toks = W.prefix_tokens(w, b, l, n)
                     _, S = O.gdn_recurrent(O.bf16_to_f64(toks["q"]), O.bf16_to_f64(toks["k"]),
                                            O.bf16_to_f64(toks["v"]), O.f32_to_f64(toks["alpha"]),
@@ -104,13 +106,38 @@ class Pair:
         other.oracle = copy.deepcopy(self.oracle)
         return other
 
-    def run_round(self, span_cu, sb, se, tails, inputs, check_bitexact=True, via="update_round"):
+    def rerotate(self, b, begin, end, new_pos):
+        """Tail-and-relocate on both sides: stored keys of live entries
+        [begin, end) of character b turned to position ids new_pos.  Returns
+        rel-L2 errors of the turned keys per attention layer; positions are
+        checked exactly."""
+        s = self.shape
+        self.ctx.rerotate_keys(b, begin, end, new_pos)
+        self.ctx.check()
+        st = self.oracle[b]
+        errs = {}
+        for l in s.attn_layers:
+            st.caches[l] = O.rerotate_keys(st.caches[l], begin, end, new_pos, s.rotary_dim, s.rope_theta)
+            k1, _ = self.ctx.get_kv(l, b)
+            errs[("rerotated_k", l, b)] = rel_l2(O.bf16_to_f64(torch_bf16_bits(k1))[:, begin:end],
+                                                 st.caches[l].K[:, begin:end])
+            assert np.array_equal(self.ctx.get_positions(b).cpu().numpy(), st.caches[l].pos.astype(np.int32))
+        st.cursor = max(st.cursor, int(np.max(new_pos)) + 1) if len(new_pos) else st.cursor
+        assert self.ctx.get_live(b)[1] == st.cursor
+        return errs
+
+    def run_round(self, span_cu, sb, se, tails, inputs, check_bitexact=True, via="update_round",
+                  tail_pos=None, delim=None):
         """One round on both sides.  Returns dict of rel-L2 errors and raises on
-        any bit-exactness violation."""
+        any bit-exactness violation.  tail_pos: optional int32 [sum M] position
+        ids of the tail (placement variants); delim: optional (cu, begins,
+        ends) of maintenance delimiters (update_round only)."""
         import torch
         s = self.shape
         B = self.B
         tail_cu = np.concatenate([[0], np.cumsum(tails)]).astype(np.int32)
+        if delim is not None:
+            assert via == "update_round", "delimiters are a field of kvm_update_round"
         pre = self.snapshot_kv() if check_bitexact else None
         L_before = [self.ctx.get_live(b)[0] for b in range(B)]
         cur_before = [self.ctx.get_live(b)[1] for b in range(B)]
@@ -130,17 +157,18 @@ class Pair:
             dev_in[l] = d
         gather = torch.full((max(1, sum(L_before)),), -1, dtype=torch.int32, device="cuda")
         if via == "update_round":
-            self.ctx.update_round(span_cu, sb, se, tail_cu, dev_in, dev_out, gather_out=gather)
+            self.ctx.update_round(span_cu, sb, se, tail_cu, dev_in, dev_out, gather_out=gather, tail_pos=tail_pos,
+                                  delim=delim)
         else:
             self.ctx.kv_compact(span_cu, sb, se, gather_out=gather)
             for l, kind in enumerate(s.layer_kind):
                 d = dev_in[l]
                 if kind == W.ATTN:
-                    self.ctx.tail_attn_prefill(l, tail_cu, d["q"], d["k"], d["v"], dev_out[l])
+                    self.ctx.tail_attn_prefill(l, tail_cu, d["q"], d["k"], d["v"], dev_out[l], tail_pos=tail_pos)
                 else:
                     self.ctx.gdn_chunk_scan_from_state(l, tail_cu, d["q"], d["k"], d["v"], d["alpha"],
                                                        d["beta"], dev_out[l])
-            self.ctx.advance(tail_cu)
+            self.ctx.advance(tail_cu, tail_pos=tail_pos)
         self.ctx.check()
         torch.cuda.synchronize()
         # ---- oracle, per character
@@ -160,16 +188,23 @@ class Pair:
                 if kind == W.GDN:
                     ins[l]["alpha"] = O.f32_to_f64(x["alpha"][t0:t1])
                     ins[l]["beta"] = O.f32_to_f64(x["beta"][t0:t1])
+            pos_b = None if tail_pos is None else np.asarray(tail_pos[t0:t1], np.int64)
+            dl_b = None
+            if delim is not None:
+                dcu, dbg, den = delim
+                dl_b = (list(dbg[dcu[b]:dcu[b + 1]]), list(den[dcu[b]:dcu[b + 1]]))
+            n_delim = 0 if dl_b is None else int(sum(e - a for a, e in zip(*dl_b)))
             outs, new = O.maintenance_round(self.oracle[b], s.layer_kind, bb, ee, ins, s.rotary_dim,
-                                            s.rope_theta)
+                                            s.rope_theta, positions=pos_b, delimiters=dl_b)
             for l in outs:
                 ora_out[l][t0:t1] = outs[l]
             self.oracle[b] = new
             # bookkeeping
             L_new = L_before[b] - int(np.sum(np.asarray(ee) - np.asarray(bb)))
             live, cur = self.ctx.get_live(b)
-            assert live == L_new + (t1 - t0), (b, live, L_new)
-            assert cur == cur_before[b] + (t1 - t0)
+            assert live == L_new + (t1 - t0) - n_delim, (b, live, L_new)
+            if tail_pos is None:
+                assert cur == cur_before[b] + (t1 - t0)
             assert new.cursor == cur
             keep_idx = np.nonzero(O.keep_mask(L_before[b], bb, ee))[0]
             assert np.array_equal(gather_np[g_off:g_off + L_new], keep_idx), f"gather map char {b}"
@@ -183,11 +218,12 @@ class Pair:
                     assert np.array_equal(k1[:, :L_new], k0[:, keep_idx]), f"K compaction layer {l} char {b}"
                     assert np.array_equal(v1[:, :L_new], v0[:, keep_idx]), f"V compaction layer {l} char {b}"
                     assert np.array_equal(p1[:L_new], p0[keep_idx]), f"positions layer {l} char {b}"
-                    assert np.array_equal(p1[L_new:], np.arange(cur_before[b], cur_before[b] + t1 - t0)), \
-                        f"tail positions char {b}"
-                    assert np.array_equal(p1, new.caches[l].pos.astype(np.int32))
+                    if tail_pos is None and delim is None:
+                        assert np.array_equal(p1[L_new:], np.arange(cur_before[b], cur_before[b] + t1 - t0)), \
+                            f"tail positions char {b}"
+                    assert np.array_equal(p1, new.caches[l].pos.astype(np.int32)), f"positions char {b}"
                     # appended rotated keys and values against the oracle's fp64 ones
-                    if t1 > t0:
+                    if new.caches[l].live > L_new:
                         errs[("append_k", l, b)] = rel_l2(O.bf16_to_f64(k1[:, L_new:]), new.caches[l].K[:, L_new:])
                         assert np.array_equal(O.bf16_to_f64(v1[:, L_new:]), new.caches[l].V[:, L_new:])
         # the bar holds per (layer, character) for outputs and per (layer,

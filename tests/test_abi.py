@@ -54,13 +54,13 @@ def _desc(kvm, kinds, **kw):
              n_gdn_heads=16, d_k=128, d_v=128)
     d.update(kw)
     return kvm.ModelDesc(len(kinds), arr, d["n_q_heads"], d["n_kv_heads"], d["head_dim"], d["rotary_dim"],
-                         d["rope_theta"], d["n_gdn_heads"], d["d_k"], d["d_v"]), arr
+                         d["rope_theta"], d["n_gdn_heads"], d["d_k"], d["d_v"], d.get("conv_kernel", 0)), arr
 
 
 @pytest.mark.parametrize("kw,code", [({"head_dim": 96}, 6), ({"n_q_heads": 12, "n_kv_heads": 5}, 6),
                                      ({"n_q_heads": 24, "n_kv_heads": 2}, 6), ({"rotary_dim": 63}, 6),
                                      ({"d_k": 96}, 6), ({"d_v": 40}, 6), ({"d_v": 160}, 6),
-                                     ({"rope_theta": -1.0}, 1)])
+                                     ({"rope_theta": -1.0}, 1), ({"conv_kernel": 3}, 6)])
 def test_create_rejects_unsupported_shapes(lib, kw, code):
     from paper_2609_18935_gb300 import kvm
     desc, keep = _desc(kvm, [0, 0, 0, 1], **kw)

@@ -231,5 +231,53 @@ def test_spans_from_positions_match_brute_force():
 
 def test_spans_from_positions_rejects_bad_positions():
     with pytest.raises(kvm.KvmError) as ei:
-        kvm.plan_spans_from_positions([3, 3, 4], [0], [5])    # not strictly increasing
+        kvm.plan_spans_from_positions([3, -1, 4], [0], [5])   # a negative position id
     assert ei.value.code == KVM_E_INVAL
+
+
+def test_spans_from_positions_out_of_order_brute_force():
+    """After slot-preserving placement or re-rotation (§5.2) live positions
+    need not increase: a range then maps to the live entries whose positions
+    lie in it, which must form one contiguous run of live indices."""
+    rng = np.random.default_rng(261955)
+    checked = 0
+    for trial in range(400):
+        live = int(rng.integers(1, 40))
+        positions = rng.choice(np.arange(200), size=live, replace=False).astype(np.int32)
+        if trial % 2:                                        # mostly increasing, one block moved back
+            positions = np.sort(positions)
+            a = int(rng.integers(0, live))
+            e = int(rng.integers(a, live)) + 1
+            positions[a:e] = np.sort(rng.choice(np.arange(1000, 1100), size=e - a, replace=False))
+        b0 = int(rng.integers(-5, 1100))
+        e0 = b0 + int(rng.integers(1, 120))
+        idx = np.flatnonzero((positions >= b0) & (positions < e0))
+        ok = idx.size > 0 and idx[-1] - idx[0] + 1 == idx.size
+        if not ok:
+            with pytest.raises(kvm.KvmError) as ei:
+                kvm.plan_spans_from_positions(positions, [b0], [e0])
+            assert ei.value.code == KVM_E_SPAN
+            continue
+        sb, se = kvm.plan_spans_from_positions(positions, [b0], [e0])
+        assert (int(sb[0]), int(se[0])) == (int(idx[0]), int(idx[-1]) + 1)
+        checked += 1
+    assert checked > 30
+
+
+def test_probe_statistics_match_the_oracle():
+    """kvm_effective_group_count and kvm_total_variation (host only) against
+    the oracle's definitions, on random masses and distributions."""
+    rng = np.random.default_rng(1832)
+    for trial in range(50):
+        n = int(rng.integers(1, 40))
+        mass = rng.random(n) * (rng.random(n) < 0.7)
+        if mass.sum() == 0:
+            mass[0] = 1.0
+        assert abs(kvm.effective_group_count(mass) - O.effective_group_count(mass)) < 1e-12
+        p, q = rng.random(n), rng.random(n)
+        p, q = p / p.sum(), q / q.sum()
+        assert abs(kvm.total_variation(p, q) - O.total_variation(p, q)) < 1e-15
+    with pytest.raises(kvm.KvmError):
+        kvm.effective_group_count([0.0, 0.0])
+    with pytest.raises(kvm.KvmError):
+        kvm.effective_group_count([0.5, -0.1])
