@@ -303,6 +303,56 @@ def gdn_chunked(q, k, v, alpha, beta, S0, C: int = 64):
 
 
 # ----------------------------------------------------------------------------
+# Short convolution of a gated-delta-rule layer (§4.1: R_t holds the
+# recurrent and the convolution states, and both continue without rollback)
+# ----------------------------------------------------------------------------
+def silu(x):
+    """x * sigmoid(x)."""
+    x = np.asarray(x, np.float64)
+    return x / (1.0 + np.exp(-x))
+
+
+def short_conv(x, state, w):
+    """Causal depthwise convolution of width 4 over a tail, continuing from
+    the carried state.
+
+    x [M][C] pre-convolution inputs of the tail; state [3][C] the last three
+    inputs before it (oldest first; zeros for a fresh context); w [C][4].
+    With xx = [state; x], output t is y_t[c] = sum_{i=0..3} w[c][i] xx[t+i][c]
+    (tap 3 is the current token).  Returns (y [M][C] before the activation,
+    the new state: the last three rows of xx)."""
+    x = np.asarray(x, np.float64)
+    w = np.asarray(w, np.float64)
+    xx = np.concatenate([np.asarray(state, np.float64), x], axis=0)
+    M = x.shape[0]
+    y = np.zeros_like(x)
+    for t in range(M):
+        for i in range(4):
+            y[t] += w[:, i] * xx[t + i]
+    return y, xx[-3:].copy()
+
+
+def gdn_conv_inputs(q, k, v, conv_state, w):
+    """Delta-rule inputs of a layer with short convolution: the channels of
+    q [M][H][d_k], k [M][H][d_k], v [M][H][d_v] (in that order) go through
+    short_conv and SiLU, then each head's k is scaled to unit L2 norm.
+    Returns (q', k', v', new conv state)."""
+    q = np.asarray(q, np.float64)
+    k = np.asarray(k, np.float64)
+    v = np.asarray(v, np.float64)
+    M, H, dk = q.shape
+    dv = v.shape[2]
+    x = np.concatenate([q.reshape(M, H * dk), k.reshape(M, H * dk), v.reshape(M, H * dv)], axis=1)
+    y, new_state = short_conv(x, conv_state, w)
+    y = silu(y)
+    q2 = y[:, :H * dk].reshape(M, H, dk)
+    k2 = y[:, H * dk:2 * H * dk].reshape(M, H, dk)
+    v2 = y[:, 2 * H * dk:].reshape(M, H, dv)
+    k2 = k2 / np.linalg.norm(k2, axis=-1, keepdims=True)
+    return q2, k2, v2, new_state
+
+
+# ----------------------------------------------------------------------------
 # Character state and one maintenance round (Eqs. 2-3)
 # ----------------------------------------------------------------------------
 class AttnCache:
@@ -323,12 +373,15 @@ class AttnCache:
 
 class CharacterState:
     """(A_t, R_t, p_t) of one character (§4.1): caches[layer] for attention
-    layers, states[layer] = S [H][d_v][d_k] for delta-rule layers, cursor p."""
+    layers, states[layer] = S [H][d_v][d_k] for delta-rule layers, cursor p;
+    conv[layer] = the short-convolution state [3][C] of delta-rule layers
+    that have one (empty otherwise)."""
 
-    def __init__(self, caches: dict, states: dict, cursor: int):
+    def __init__(self, caches: dict, states: dict, cursor: int, conv: dict | None = None):
         self.caches = caches
         self.states = states
         self.cursor = int(cursor)
+        self.conv = dict(conv) if conv else {}
 
     @classmethod
     def empty(cls, layer_kind, Hkv, D, H, dk, dv):
@@ -344,7 +397,7 @@ class CharacterState:
     def copy(self):
         return CharacterState({l: c.copy() for l, c in self.caches.items()},
                               {l: s.copy() for l, s in self.states.items()},
-                              self.cursor)
+                              self.cursor, {l: c.copy() for l, c in self.conv.items()})
 
 
 def tail_attn_prefill(cache: AttnCache, q, k_new, v_new, p: int, R: int, theta: float, positions=None):
@@ -384,7 +437,8 @@ def rerotate_keys(cache: AttnCache, begin: int, end: int, new_pos, R: int, theta
 
 
 def maintenance_round(state: CharacterState, layer_kind, begins, ends,
-                      inputs: dict, R: int, theta: float, positions=None, delimiters=None):
+                      inputs: dict, R: int, theta: float, positions=None, delimiters=None,
+                      conv_weights: dict | None = None):
     """One round for one character: Eq. 2 on every attention layer, then
     Eq. 3 layer by layer in model order, then p += M.
 
@@ -396,6 +450,9 @@ def maintenance_round(state: CharacterState, layer_kind, begins, ends,
     direct KV are removed from every attention layer; their effect on the
     recurrent states and on later tail tokens remains, and their position
     ids stay consumed.
+    conv_weights: optional {layer: w [C][4]} of delta-rule layers with short
+    convolution; their q/k/v inputs are then pre-convolution projections,
+    convolved from state.conv[layer] (zeros if absent) by gdn_conv_inputs.
     Returns (outputs {layer: [M][heads][dim]}, new state).  `state` is not
     modified."""
     new = state.copy()
@@ -413,8 +470,12 @@ def maintenance_round(state: CharacterState, layer_kind, begins, ends,
             outs[l], new.caches[l] = tail_attn_prefill(new.caches[l], x["q"], x["k"], x["v"],
                                                        new.cursor, R, theta, positions)
         else:
-            outs[l], new.states[l] = gdn_recurrent(x["q"], x["k"], x["v"], x["alpha"],
-                                                   x["beta"], new.states[l])
+            q, k, v = x["q"], x["k"], x["v"]
+            if conv_weights is not None and l in conv_weights:
+                w = np.asarray(conv_weights[l], np.float64)
+                st0 = new.conv.get(l, np.zeros((3, w.shape[0])))
+                q, k, v, new.conv[l] = gdn_conv_inputs(q, k, v, st0, w)
+            outs[l], new.states[l] = gdn_recurrent(q, k, v, x["alpha"], x["beta"], new.states[l])
     if M is not None:
         if positions is None:
             new.cursor += M
@@ -432,8 +493,8 @@ def maintenance_round(state: CharacterState, layer_kind, begins, ends,
     return outs, new
 
 
-def refill(layer_kind, inputs: dict, Hkv, D, H, dk, dv, R, theta):
+def refill(layer_kind, inputs: dict, Hkv, D, H, dk, dv, R, theta, conv_weights=None):
     """Dense refill: the whole token sequence read from an empty state at
     positions 0 .. n-1 (the reference construction of §5.2)."""
     empty = CharacterState.empty(layer_kind, Hkv, D, H, dk, dv)
-    return maintenance_round(empty, layer_kind, [], [], inputs, R, theta)
+    return maintenance_round(empty, layer_kind, [], [], inputs, R, theta, conv_weights=conv_weights)

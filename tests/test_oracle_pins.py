@@ -696,3 +696,78 @@ def test_total_variation_is_the_largest_event_difference():
         assert abs(O.total_variation(p, q) - best) < 1e-12
     assert O.total_variation([1, 0], [0, 1]) == 1.0
     assert O.total_variation([0.3, 0.7], [0.3, 0.7]) == 0.0
+
+
+# ---------------------------------------------------------------- short convolution (§4.1)
+def test_short_conv_from_zero_state_is_numpy_convolution():
+    """From a zero state the carried convolution is the causal part of the
+    full convolution with the reversed taps (numpy's convolve)."""
+    M, C = 11, 5
+    x = rng.standard_normal((M, C))
+    w = rng.standard_normal((C, 4))
+    y, st = O.short_conv(x, np.zeros((3, C)), w)
+    for c in range(C):
+        np.testing.assert_allclose(y[:, c], np.convolve(x[:, c], w[c, ::-1])[:M], atol=1e-12)
+    np.testing.assert_array_equal(st, x[-3:])
+
+
+def test_short_conv_state_carry_equals_one_pass():
+    """Rounds of 5, 1, 2 and 7 tokens, each continuing from the state the
+    previous one left, give the convolution of the whole sequence (numpy's
+    convolve), and the state is always the last three inputs."""
+    C = 4
+    x = rng.standard_normal((15, C))
+    w = rng.standard_normal((C, 4))
+    st = np.zeros((3, C))
+    parts, at = [], 0
+    for m in (5, 1, 2, 7):
+        y, st = O.short_conv(x[at:at + m], st, w)
+        parts.append(y)
+        at += m
+        seen = np.concatenate([np.zeros((3, C)), x[:at]])
+        np.testing.assert_array_equal(st, seen[-3:])
+    y = np.concatenate(parts)
+    for c in range(C):
+        np.testing.assert_allclose(y[:, c], np.convolve(x[:, c], w[c, ::-1])[:15], atol=1e-12)
+
+
+def test_silu_and_identity_taps():
+    from scipy.special import expit
+    x = rng.standard_normal(50) * 4
+    np.testing.assert_allclose(O.silu(x), x * expit(x), atol=1e-12)
+    assert O.silu(0.0) == 0.0
+    w = np.tile([0.0, 0.0, 0.0, 1.0], (3, 1))            # only the current token
+    q = rng.standard_normal((6, 1, 1))
+    k = rng.standard_normal((6, 1, 1))
+    v = rng.standard_normal((6, 1, 1))
+    q2, k2, v2, st = O.gdn_conv_inputs(q, k, v, rng.standard_normal((3, 3)), w)
+    np.testing.assert_allclose(q2, O.silu(q), atol=1e-12)
+    np.testing.assert_allclose(v2, O.silu(v), atol=1e-12)
+    np.testing.assert_allclose(np.abs(k2), 1.0, atol=1e-12)   # d_k = 1: unit norm is +-1
+    np.testing.assert_array_equal(st[:, 0], q[-3:, 0, 0])
+
+
+def test_zero_removal_tail_update_equals_refill_with_conv_state():
+    """The refill equivalence (causality) holds with the convolution state
+    carried across the round boundary: outputs, S and conv state."""
+    st = _stack()
+    N, M = 17, 9
+    ins = _tokens(N + M, st)
+    Cch = st["H"] * (2 * st["dk"] + st["dv"])
+    convw = {l: rng.standard_normal((Cch, 4)) * 0.5 for l, kd in enumerate(st["layer_kind"]) if kd == 0}
+    args = (st["Hkv"], st["D"], st["H"], st["dk"], st["dv"], st["R"], st["theta"])
+    _, pre = O.refill(st["layer_kind"], _cut(ins, 0, N), *args, conv_weights=convw)
+    outs, post = O.maintenance_round(pre, st["layer_kind"], [], [], _cut(ins, N, N + M), st["R"], st["theta"],
+                                     conv_weights=convw)
+    ref_outs, ref = O.refill(st["layer_kind"], ins, *args, conv_weights=convw)
+    for l in outs:
+        np.testing.assert_allclose(outs[l], ref_outs[l][N:], atol=1e-12)
+    for l in post.states:
+        np.testing.assert_allclose(post.states[l], ref.states[l], atol=1e-12)
+        np.testing.assert_array_equal(post.conv[l], ref.conv[l])
+    # without carrying the conv state (restarting it from zero) the outputs differ
+    cold = pre.copy()
+    cold.conv = {}
+    o_cold, _ = O.maintenance_round(cold, st["layer_kind"], [], [], _cut(ins, N, N + M), st["R"], st["theta"],
+                                    conv_weights=convw)
+    assert not np.allclose(o_cold[0][:3], outs[0][:3])
