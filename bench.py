@@ -270,6 +270,23 @@ def replica_seed(rank: int) -> int:
     return 7919 * (rank + 1)
 
 
+def rank_share(w, rank: int, world: int):
+    """The characters rank `rank` maintains.  A population (several
+    characters) is partitioned over the ranks by kvm_plan_partition, balanced
+    by each character's round-0 attention work M (L' + (M + 1) / 2); the
+    ranks need no exchange on the data path, and the job's total work stays
+    fixed as ranks are added (strong scaling).  A single character cannot be
+    split: every rank maintains its own replica (weak scaling).
+    Returns (workload of this rank, scaling)."""
+    if world <= 1 or w.n_chars <= 1:
+        return w, "weak"
+    from paper_2609_18935_gb300 import kvm
+    cu, sb, se, tails = W.round_plan(w, 0, list(w.prefix_len))
+    after = [w.prefix_len[b] - int((se[cu[b]:cu[b + 1]] - sb[cu[b]:cu[b + 1]]).sum()) for b in range(w.n_chars)]
+    rank_of, _ = kvm.plan_partition(kvm.round_cost(after, tails), world)
+    return w.subset([b for b in range(w.n_chars) if rank_of[b] == rank]), "strong"
+
+
 def max_over_ranks(x: float, world: int, device="cpu") -> float:
     """The job's time is the slowest rank's (all_reduce MAX); x itself on one rank."""
     if world <= 1:
@@ -281,6 +298,17 @@ def max_over_ranks(x: float, world: int, device="cpu") -> float:
     return float(t.item())
 
 
+def sum_over_ranks(x: float, world: int, device="cpu") -> float:
+    """Sum of x over the ranks (all_reduce SUM); x itself on one rank."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
 def job_throughput(world: int, tokens_per_rank: float, ms: float) -> float:
     """Whole-job tail tokens/s: every rank processes tokens_per_rank in the
     job's time (the slowest rank's) of ms milliseconds."""
@@ -289,10 +317,15 @@ def job_throughput(world: int, tokens_per_rank: float, ms: float) -> float:
 
 def workload_config(w, args, world):
     s = w.shape
-    return {"workload": WORKLOAD_TEXT[args.workload], "name": args.workload, "chars": w.n_chars,
+    full = W.make_workload(args.workload)
+    if world > 1 and full.n_chars > 1:
+        par = f"population of {full.n_chars} characters partitioned over {world} ranks (balanced by M L')"
+    else:
+        par = f"{world} independent replica(s), characters per rank fixed"
+    return {"workload": WORKLOAD_TEXT[args.workload], "name": args.workload, "chars": full.n_chars,
             "layers": len(s.layer_kind), "chain_rounds": w.rounds,
             "l2": "flushed before every step (256 MiB write), outside the timed events",
-            "parallelism": f"{world} independent replica(s), characters per rank fixed"}
+            "parallelism": par}
 
 
 def run_reference(args):
@@ -376,7 +409,7 @@ def run_kvm(args):
             dist.barrier()
     kvm.load_library()
 
-    w = W.make_workload(args.workload)
+    w, scaling = rank_share(W.make_workload(args.workload), rank, world)
     s = w.shape
     plan = W.simulate_plan(w)
     R = len(plan)
@@ -500,9 +533,12 @@ def run_kvm(args):
     scratch = from_scratch_prefill(w, plan, mk, flush, args, seed_base) if args.workload == "refill" else None
     clocks.stop()
 
-    toks_rank = sum(sum(rounds[r]["tails"]) for r in rids)
-    value = job_throughput(world, toks_rank, total_ms)
-    e2e_value = job_throughput(world, sum(sum(rounds[r]["tails"]) for r in e2e_rids), e2e_ms)
+    # every rank's tail tokens over the job's time (replicas process equal
+    # shares; a partitioned population does not)
+    toks_job = sum_over_ranks(float(sum(sum(rounds[r]["tails"]) for r in rids)), world, device="cuda")
+    value = job_throughput(1, toks_job, total_ms)
+    e2e_value = job_throughput(1, sum_over_ranks(float(sum(sum(rounds[r]["tails"]) for r in e2e_rids)), world,
+                                                 device="cuda"), e2e_ms)
     hbm, tc_burst, tc_sust, peak_src = load_peaks()
     n_attn, n_gdn = len(s.attn_layers), len(s.gdn_layers)
     # algorithmic work of every kernel family over the steps of the per-kernel pass
@@ -573,7 +609,7 @@ def run_kvm(args):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "scaling": scaling, "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": workload_config(w, args, world),
         "roofline": roofline,
         "round_roofline": round_roofline,

@@ -204,6 +204,19 @@ kvm_status kvm_plan_attention(int32_t n_chars, const int32_t* live, const int32_
                               int32_t* n_blocks, int32_t* n_tiles, int32_t* block_tile,
                               int32_t* block_key, int32_t* n_split, int32_t* split_first_block);
 
+/* Partition of a character population over ranks (one GPU per rank):
+ * characters are independent, so each rank maintains its own share with no
+ * exchange on the data path.  cost host [n_chars] >= 0, e.g. a round's
+ * attention work M_b (L'_b + (M_b + 1) / 2), the term the round's time
+ * follows.  Longest-processing-time first: characters by decreasing cost
+ * (ties by index), each to the rank with the least cost so far (ties: the
+ * lowest rank), so the heaviest rank exceeds the mean by less than the
+ * largest single cost.  rank_of host [n_chars]; rank_cost host [n_ranks]
+ * (may be NULL).  Deterministic: every rank computes the same plan.
+ * Errors: KVM_E_INVAL. */
+kvm_status kvm_plan_partition(int32_t n_chars, const int64_t* cost, int32_t n_ranks, int32_t* rank_of,
+                              int64_t* rank_cost);
+
 /* ------------------------------------------------------------ hot path */
 
 /* Eq. 2: remove the live entries named by the spans from every attention

@@ -755,6 +755,29 @@ extern "C" kvm_status kvm_plan_attention(int32_t n_chars, const int32_t* live, c
     return KVM_OK;
 }
 
+extern "C" kvm_status kvm_plan_partition(int32_t n_chars, const int64_t* cost, int32_t n_ranks, int32_t* rank_of,
+                                         int64_t* rank_cost) {
+    if (n_chars < 0 || n_ranks < 1) return fail(KVM_E_INVAL, "need n_chars >= 0 and n_ranks >= 1");
+    if (n_chars > 0 && (!cost || !rank_of)) return fail(KVM_E_INVAL, "NULL argument");
+    for (int b = 0; b < n_chars; ++b)
+        if (cost[b] < 0) return fail(KVM_E_INVAL, "cost of character %d is negative", b);
+    // longest processing time first: characters by decreasing cost (ties by
+    // index), each to the rank with the least cost so far (ties: lowest rank)
+    std::vector<int> order(n_chars);
+    for (int b = 0; b < n_chars; ++b) order[b] = b;
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return cost[a] > cost[b]; });
+    std::vector<int64_t> load(n_ranks, 0);
+    for (int b : order) {
+        int best = 0;
+        for (int r = 1; r < n_ranks; ++r)
+            if (load[r] < load[best]) best = r;
+        rank_of[b] = best;
+        load[best] += cost[b];
+    }
+    if (rank_cost) std::copy(load.begin(), load.end(), rank_cost);
+    return KVM_OK;
+}
+
 namespace {
 // Position ranges -> live-index spans over the live positions P[live].
 // Positions are in live order; they increase unless per-token positions or

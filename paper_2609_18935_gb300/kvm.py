@@ -91,6 +91,8 @@ _SIGS = {
     "kvm_plan_attention": (C.c_int, [C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.c_int32, C.c_int32,
                                      C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32),
                                      C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32)]),
+    "kvm_plan_partition": (C.c_int, [C.c_int32, C.POINTER(C.c_int64), C.c_int32, C.POINTER(C.c_int32),
+                                     C.POINTER(C.c_int64)]),
     "kvm_kv_compact_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int64, C.c_int32,
                                          C.c_int32, C.c_int32, C.POINTER(C.c_int32), C.POINTER(C.c_int32),
                                          C.POINTER(C.c_int32), C.c_void_p]),
@@ -262,6 +264,24 @@ def plan_attention(live, tail_cu, n_q_heads, n_kv_heads, max_blocks):
     n = nb.value
     return {"n_blocks": n, "n_tiles": nt.value, "block_tile": tile[:n + 1].copy(), "block_key": key[:n + 1].copy(),
             "split_first_block": split[:ns.value].copy()}
+
+
+def round_cost(live_after_removal, tails):
+    """Per-character cost of a round's attention, M_b (L'_b + (M_b + 1) / 2),
+    in units of query-key pairs (the partitioner's balance target)."""
+    return [int(m) * int(l) + int(m) * (int(m) + 1) // 2 for l, m in zip(live_after_removal, tails)]
+
+
+def plan_partition(cost, n_ranks):
+    """kvm_plan_partition: (rank of each character, summed cost per rank)."""
+    load_library()
+    c = np.ascontiguousarray(np.asarray(cost, dtype=np.int64))
+    rank_of = np.zeros(len(c), np.int32)
+    loads = np.zeros(int(n_ranks), np.int64)
+    p64 = lambda a: a.ctypes.data_as(C.POINTER(C.c_int64))
+    _check(_lib.kvm_plan_partition(len(c), p64(c) if len(c) else None, int(n_ranks),
+                                   _p32(rank_of) if len(c) else None, p64(loads)))
+    return rank_of, loads
 
 
 def pinned_layer_inputs(inputs):

@@ -38,14 +38,28 @@ class Pair:
     """A GPU context and per-character oracle states holding the same prefix."""
 
     def __init__(self, shape: W.ModelShape, prefix_len, capacity, max_tail, seed_index=0,
-                 prefix="random", cursor_offset=0):
+                 prefix="random", cursor_offset=0, conv=False):
         import torch
         from paper_2609_18935_gb300 import kvm
         self.shape = shape
         s = shape
+        ck = 4 if conv else 0
         self._new_ctx = lambda: kvm.Context(s.layer_kind, s.n_q_heads, s.n_kv_heads, s.head_dim, s.rotary_dim,
-                                            s.rope_theta, s.n_gdn_heads, s.d_k, s.d_v, capacity, max_tail)
+                                            s.rope_theta, s.n_gdn_heads, s.d_k, s.d_v, capacity, max_tail,
+                                            conv_kernel=ck)
         self.ctx = self._new_ctx()
+        # short convolution: taps per delta-rule layer and a random carried
+        # state (the last three pre-convolution inputs of an earlier round)
+        self.conv_w = None
+        conv_state = {}
+        if conv:
+            C_ = s.n_gdn_heads * (2 * s.d_k + s.d_v)
+            self.conv_w = {l: W.conv_weights((seed_index, 996, l), C_) for l in s.gdn_layers}
+            for l in s.gdn_layers:
+                bits = W.normal_bf16((seed_index, 995, l), (len(prefix_len), 3, C_))
+                conv_state[l] = bits
+                self.ctx.set_conv_weights(l, torch.from_numpy(self.conv_w[l]).cuda())
+                self.ctx.set_conv_state(l, to_torch_bf16(bits).cuda())
         self.B = len(prefix_len)
         self.oracle = []
         w = W.Workload("custom", seed_index, shape, list(prefix_len), 1)
@@ -79,7 +93,8 @@ class Pair:
                     S32 = W.prefix_state(w, b, l)
                 S_all[l][b] = S32
                 states[l] = O.f32_to_f64(S32)
-            self.oracle.append(O.CharacterState(caches, states, cursor))
+            self.oracle.append(O.CharacterState(caches, states, cursor,
+                                                {l: O.bf16_to_f64(conv_state[l][b]) for l in conv_state}))
         for l in s.gdn_layers:
             self.ctx.set_state(l, torch.from_numpy(S_all[l]).cuda())
         torch.cuda.synchronize()
@@ -195,7 +210,8 @@ class Pair:
                 dl_b = (list(dbg[dcu[b]:dcu[b + 1]]), list(den[dcu[b]:dcu[b + 1]]))
             n_delim = 0 if dl_b is None else int(sum(e - a for a, e in zip(*dl_b)))
             outs, new = O.maintenance_round(self.oracle[b], s.layer_kind, bb, ee, ins, s.rotary_dim,
-                                            s.rope_theta, positions=pos_b, delimiters=dl_b)
+                                            s.rope_theta, positions=pos_b, delimiters=dl_b,
+                                            conv_weights=self.conv_w)
             for l in outs:
                 ora_out[l][t0:t1] = outs[l]
             self.oracle[b] = new
@@ -234,6 +250,12 @@ class Pair:
                 t0, t1 = tail_cu[b], tail_cu[b + 1]
                 if t1 > t0:
                     errs[("out", l, b)] = rel_l2(gpu_out[l][t0:t1], ora_out[l][t0:t1])
+        if self.conv_w is not None:
+            # the carried conv state holds raw bf16 inputs: bit-exact
+            for l in s.gdn_layers:
+                cs = O.bf16_to_f64(torch_bf16_bits(self.ctx.get_conv_state(l)))
+                for b in range(B):
+                    assert np.array_equal(cs[b], self.oracle[b].conv[l]), f"conv state layer {l} char {b}"
         for l in s.gdn_layers:
             S_gpu = self.ctx.get_state(l).cpu().numpy().astype(np.float64)
             for b in range(B):

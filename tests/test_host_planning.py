@@ -281,3 +281,26 @@ def test_probe_statistics_match_the_oracle():
         kvm.effective_group_count([0.0, 0.0])
     with pytest.raises(kvm.KvmError):
         kvm.effective_group_count([0.5, -0.1])
+
+
+def test_partition_balance_and_brute_force():
+    """kvm_plan_partition: each character on exactly one rank, the heaviest
+    rank within the largest cost of the mean (the LPT bound), and within 4/3
+    of the best partition found by enumeration on small populations."""
+    import itertools
+    rng = np.random.default_rng(31)
+    for trial in range(60):
+        n = int(rng.integers(1, 9))
+        ranks = int(rng.integers(1, 4))
+        cost = [int(x) for x in rng.integers(0, 10_000, size=n)]
+        rank_of, loads = kvm.plan_partition(cost, ranks)
+        assert len(rank_of) == n and all(0 <= r < ranks for r in rank_of)
+        got = [sum(c for c, r in zip(cost, rank_of) if r == k) for k in range(ranks)]
+        assert got == list(loads)
+        assert max(got) <= sum(cost) / ranks + max(cost)
+        best = min(max(sum(c for c, r in zip(cost, a) if r == k) for k in range(ranks))
+                   for a in itertools.product(range(ranks), repeat=n))
+        assert max(got) <= best * 4 / 3 + 1e-9
+    assert list(kvm.plan_partition([5, 5, 5, 5], 2)[1]) == [10, 10]
+    with pytest.raises(kvm.KvmError):
+        kvm.plan_partition([1, -2], 2)

@@ -83,6 +83,13 @@ def gates(seed: tuple, n: int, heads: int):
     return a, b
 
 
+def conv_weights(seed: tuple, channels: int, std: float = 0.5) -> np.ndarray:
+    """Short-convolution taps of a delta-rule layer, fp32 [channels][4],
+    N(0, std^2) (four taps of std 0.5 keep the pre-activation near unit
+    scale for unit-scale inputs)."""
+    return (_rng(*seed).standard_normal((channels, 4)) * std).astype(np.float32)
+
+
 def state_f32(seed: tuple, shape, std: float = 0.2) -> np.ndarray:
     return (_rng(*seed).standard_normal(shape) * std).astype(np.float32)
 
@@ -166,10 +173,26 @@ class Workload:
     # per round, per character: (removal fraction, number of spans, tail M)
     plan: list = field(default_factory=list)
     refill_compare: bool = False
+    # population index of each character (its seeds); None: 0 .. n_chars-1.
+    # A rank's share of a partitioned population keeps its characters' ids,
+    # so they draw the same numbers as in the whole population.
+    char_ids: list | None = None
 
     @property
     def n_chars(self):
         return len(self.prefix_len)
+
+    def gid(self, b: int) -> int:
+        return b if self.char_ids is None else int(self.char_ids[b])
+
+    def subset(self, chars) -> "Workload":
+        """The workload restricted to characters `chars` (population indices
+        in order), with their plans and seeds."""
+        chars = [int(b) for b in chars]
+        sub = Workload(self.name, self.index, self.shape, [self.prefix_len[b] for b in chars], self.rounds,
+                       [[row[b] for b in chars] for row in self.plan], self.refill_compare,
+                       [self.gid(b) for b in chars])
+        return sub
 
     def capacity(self, align: int = 128) -> list:
         """Slots per character that hold the prefix plus every tail of the
@@ -241,7 +264,7 @@ def tail_inputs(w: Workload, rnd: int, tails: list, layers=None) -> dict:
             continue
         parts = {"q": [], "k": [], "v": [], "alpha": [], "beta": []}
         for b, m in enumerate(tails):
-            sd = (base, b, layer)
+            sd = (base, w.gid(b), layer)
             if kind == ATTN:
                 parts["q"].append(normal_bf16(sd + (0,), (m, s.n_q_heads, s.head_dim)))
                 parts["k"].append(normal_bf16(sd + (1,), (m, s.n_kv_heads, s.head_dim), unit_last=True))
@@ -266,7 +289,7 @@ def round_plan(w: Workload, rnd: int, live: list):
     for b, L in enumerate(live):
         frac, n_sp, m = w.plan[rnd][b]
         total = int(round(frac * L))
-        bb, ee = removal_spans((w.index * 1000 + rnd, b, 7777), L, total, n_sp)
+        bb, ee = removal_spans((w.index * 1000 + rnd, w.gid(b), 7777), L, total, n_sp)
         bs.append(bb)
         es.append(ee)
         cu.append(cu[-1] + len(bb))
@@ -278,7 +301,7 @@ def round_plan(w: Workload, rnd: int, live: list):
 def prefix_tokens(w: Workload, b: int, layer: int, n: int) -> dict:
     """Raw (unrotated) prefix tokens of character b for a refill."""
     s = w.shape
-    sd = (w.index * 1000 + 999, b, layer)
+    sd = (w.index * 1000 + 999, w.gid(b), layer)
     if s.layer_kind[layer] == ATTN:
         return {"q": normal_bf16(sd + (0,), (n, s.n_q_heads, s.head_dim)),
                 "k": normal_bf16(sd + (1,), (n, s.n_kv_heads, s.head_dim), unit_last=True),
@@ -295,7 +318,7 @@ def prefix_cache(w: Workload, b: int, layer: int, n: int):
     bf16 vectors (already in stored, rotated form), values N(0,1) bf16,
     positions 0..n-1.  Shapes K,V [Hkv][n][D]."""
     s = w.shape
-    sd = (w.index * 1000 + 998, b, layer)
+    sd = (w.index * 1000 + 998, w.gid(b), layer)
     K = normal_bf16(sd + (0,), (s.n_kv_heads, n, s.head_dim), unit_last=True)
     V = normal_bf16(sd + (1,), (s.n_kv_heads, n, s.head_dim))
     return K, V, np.arange(n, dtype=np.int32)
@@ -303,7 +326,7 @@ def prefix_cache(w: Workload, b: int, layer: int, n: int):
 
 def prefix_state(w: Workload, b: int, layer: int) -> np.ndarray:
     s = w.shape
-    return state_f32((w.index * 1000 + 997, b, layer), (s.n_gdn_heads, s.d_v, s.d_k))
+    return state_f32((w.index * 1000 + 997, w.gid(b), layer), (s.n_gdn_heads, s.d_v, s.d_k))
 
 
 # ----------------------------------------------------------------------------
