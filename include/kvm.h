@@ -463,6 +463,14 @@ kvm_status kvm_check(kvm_ctx* ctx, void* stream);
  * without a fault.  Errors: KVM_E_INVAL. */
 kvm_status kvm_debug_compact_wait(kvm_ctx* ctx, int32_t polls, int32_t stall);
 
+/* Debug builds (compiled with -DKVM_DEBUG) surround every device buffer of
+ * a context with canary bands, which kvm_check verifies (KVM_E_DEVICE names
+ * the buffer whose band changed).  This call overwrites one byte just past
+ * the context's first buffer, so that tests can exercise that check without
+ * a faulty kernel.  Release builds: KVM_E_UNSUPPORTED.  No paper
+ * counterpart. */
+kvm_status kvm_debug_poke_canary(kvm_ctx* ctx);
+
 /* Number of kernel launches the library has enqueued since creation
  * (diagnostics for the benchmark). */
 int64_t kvm_launch_count(const kvm_ctx* ctx);

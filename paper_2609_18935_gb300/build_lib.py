@@ -37,30 +37,38 @@ def _run(cmd):
     return r.stdout + r.stderr
 
 
-def build(verbose_ptxas: bool = False, force: bool = False) -> str:
-    os.makedirs(BUILD, exist_ok=True)
+DEBUG_LIB = os.path.join(BUILD, "debug", "libkvm_debug.so")
+
+
+def build(verbose_ptxas: bool = False, force: bool = False, debug: bool = False) -> str:
+    """Build libkvm.so, or with `debug` the canary-checking variant
+    _build/debug/libkvm_debug.so (-DKVM_DEBUG: every device buffer of a
+    context between two canary bands that kvm_check verifies)."""
+    out_dir = os.path.dirname(DEBUG_LIB) if debug else BUILD
+    lib = DEBUG_LIB if debug else LIB
+    os.makedirs(out_dir, exist_ok=True)
     nvcc = _nvcc()
     deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC)] + \
            [os.path.join(PKG, "..", "include", "kvm.h")]
     newest_src = max(os.path.getmtime(p) for p in deps)
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= newest_src:
-        return LIB
-    extra = ["-Xptxas", "-v"] if verbose_ptxas else []
+    if not force and os.path.exists(lib) and os.path.getmtime(lib) >= newest_src:
+        return lib
+    extra = (["-Xptxas", "-v"] if verbose_ptxas else []) + (["-DKVM_DEBUG"] if debug else [])
 
     def compile_one(src):
-        obj = os.path.join(BUILD, src.replace(".cu", ".o"))
+        obj = os.path.join(out_dir, src.replace(".cu", ".o"))
         out = _run([nvcc, *ARCH, *FLAGS, *extra, "-c", os.path.join(CSRC, src), "-o", obj])
         return obj, out
 
     with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         results = list(ex.map(compile_one, SOURCES))
     logs = "".join(o for _, o in results)
-    tmp = LIB + ".tmp"
+    tmp = lib + ".tmp"
     _run([nvcc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *[o for o, _ in results]])
-    os.replace(tmp, LIB)
+    os.replace(tmp, lib)
     if verbose_ptxas:
         sys.stdout.write(logs)
-    return LIB
+    return lib
 
 
 if __name__ == "__main__":

@@ -16,6 +16,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/kvm.h"
 #include "kvm_internal.cuh"
 #include "tma_host.h"
@@ -134,6 +136,10 @@ struct kvm_ctx {
     int rows_kv = 0, rows_pos = 0;
     int compact_wait_limit = kCompactWaitLimit;   // polls of a compaction read flag before giving up
     bool compact_stall = false;                   // failure-detection tests: wait on a word nothing sets
+    // every device buffer the context owns: allocation base, user bytes, name
+    // (with KVM_DEBUG the user bytes sit between two canary bands)
+    struct DevAlloc { void* base; size_t bytes; const char* name; };
+    std::vector<DevAlloc> allocs;
     // per-kernel timing (kvm_profile_*)
     bool prof = false;
     std::vector<cudaEvent_t> ev;          // 2 per timed launch
@@ -142,27 +148,42 @@ struct kvm_ctx {
 
 namespace {
 
+// Debug builds (-DKVM_DEBUG) put a band of kCanaryByte before and after
+// every device buffer of a context; kvm_check reads the bands back and
+// reports a kernel that wrote outside its buffers as KVM_E_DEVICE.
+#ifdef KVM_DEBUG
+constexpr size_t kCanary = 4096;        // keeps the user pointer 256-byte aligned
+#else
+constexpr size_t kCanary = 0;
+#endif
+constexpr unsigned char kCanaryByte = 0xA5;
+
+// One device buffer of `count` T, zeroed (or not), registered for release
+// and for the canary check.
 template <typename T>
-cudaError_t alloc_zero(T** p, size_t count) {
-    if (count == 0) { *p = nullptr; return cudaSuccess; }
-    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T));
+cudaError_t alloc_dev(kvm_ctx* c, T** p, size_t count, const char* name, bool zero = true) {
+    *p = nullptr;
+    if (count == 0) return cudaSuccess;
+    const size_t bytes = count * sizeof(T);
+    void* base = nullptr;
+    cudaError_t e = cudaMalloc(&base, bytes + 2 * kCanary);
     if (e != cudaSuccess) return e;
-    return cudaMemset(*p, 0, count * sizeof(T));
+    c->allocs.push_back({base, bytes, name});
+    char* user = static_cast<char*>(base) + kCanary;
+    if (kCanary) {
+        e = cudaMemset(base, kCanaryByte, kCanary);
+        if (e == cudaSuccess) e = cudaMemset(user + bytes, kCanaryByte, kCanary);
+        if (e != cudaSuccess) return e;
+    }
+    *p = reinterpret_cast<T*>(user);
+    return zero ? cudaMemset(user, 0, bytes) : cudaSuccess;
 }
 
+#define alloc_zero(pp, count) alloc_dev(c, pp, count, #pp)
+
 void free_all(kvm_ctx* c) {
-    void* ptrs[] = {c->K, c->V, c->pos, c->S, c->q_rot, c->part_o, c->part_ml, c->tickets,
-                    c->flags, c->err, c->stage, c->gdn_work, c->diag};
-    for (void* p : ptrs)
-        if (p) cudaFree(p);
-    if (c->tail_pos_dev) cudaFree(c->tail_pos_dev);
-    if (c->probe_q) cudaFree(c->probe_q);
-    if (c->conv_w) cudaFree(c->conv_w);
-    if (c->conv_state) cudaFree(c->conv_state);
-    if (c->conv_y) cudaFree(c->conv_y);
-    if (c->probe_part) cudaFree(c->probe_part);
-    if (c->probe_rows) cudaFree(c->probe_rows);
-    if (c->reloc_pos_dev) cudaFree(c->reloc_pos_dev);
+    for (const auto& a : c->allocs) cudaFree(a.base);
+    c->allocs.clear();
     if (c->pos_host) cudaFreeHost(c->pos_host);
     if (c->ev_pos) cudaEventDestroy(c->ev_pos);
     for (cudaEvent_t e : c->ev_in) if (e) cudaEventDestroy(e);
@@ -486,7 +507,7 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         // one record per (64-token chunk, head); a character's tail adds at most one ragged chunk
         c->gdn_rec = gdn_record_bytes(c->dk, c->dv);
         const size_t chunks = (size_t)max_tail_tokens / 64 + n_chars;
-        if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&c->gdn_work), chunks * c->H * c->gdn_rec);
+        if (e == cudaSuccess) e = alloc_dev(c, &c->gdn_work, chunks * c->H * c->gdn_rec, "gdn_work", false);
     }
     {
         size_t total_stage = 0;
@@ -501,7 +522,7 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
             c->stage_in_off.push_back(attn ? 0 : take(T * c->H * 4));                        // beta
             c->stage_out_off.push_back(take(T * (attn ? c->Hq * c->D : c->H * c->dv) * 2));  // out
         }
-        if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&c->stage), total_stage);
+        if (e == cudaSuccess) e = alloc_dev(c, &c->stage, total_stage, "stage", false);
         if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_start, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_copies, cudaEventDisableTiming);
@@ -1314,7 +1335,23 @@ extern "C" kvm_status kvm_advance_at(kvm_ctx* c, const int32_t* tail_cu, const i
 
 extern "C" kvm_status kvm_advance(kvm_ctx* c, const int32_t* tail_cu) { return kvm_advance_at(c, tail_cu, nullptr); }
 
+namespace {
+// NVTX ranges (a tool such as Nsight Systems shows them; without one attached
+// each push / pop is a few nanoseconds).  Popped on every return path.
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
+}  // namespace
+
+kvm_status update_round_impl(kvm_ctx* c, const kvm_round* r, void* stream);
+
 extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* stream) {
+    NvtxRange range("kvm_update_round");
+    return update_round_impl(c, r, stream);
+}
+
+kvm_status update_round_impl(kvm_ctx* c, const kvm_round* r, void* stream) {
     if (!c || !r) return fail(KVM_E_INVAL, "NULL argument");
     cudaStream_t s = (cudaStream_t)stream;
     int total = 0;
@@ -1422,6 +1459,7 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
             CUDA_TRY(cudaEventRecord(c->ev_round, s));
             CUDA_TRY(cudaStreamWaitEvent(cs, c->ev_round, 0));
         }
+        NvtxRange range("kv_compact");
         // the gather map depends on the plan only; it goes first so that the
         // events of the compactions cover it
         st = launch_gather(c, pl, r->gather_out, cs);
@@ -1460,9 +1498,14 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
             }
             out = c->stage + c->stage_out_off[l];
         }
-        st = attn ? do_attention(c, l, r->tail_cu, q, k, v, out, s, with_pos ? c->tail_pos_dev : nullptr,
-                                 with_pos ? r->tail_pos : nullptr)
-                  : do_gdn(c, l, r->tail_cu, q, k, v, al, be, out, s);
+        {
+            char name[48];
+            snprintf(name, sizeof name, "layer %d (%s)", l, attn ? "attention" : "delta rule");
+            NvtxRange range(name);
+            st = attn ? do_attention(c, l, r->tail_cu, q, k, v, out, s, with_pos ? c->tail_pos_dev : nullptr,
+                                     with_pos ? r->tail_pos : nullptr)
+                      : do_gdn(c, l, r->tail_cu, q, k, v, al, be, out, s);
+        }
         if (st) {
             join();                                   // s still covers the compaction
             return st;
@@ -1506,9 +1549,42 @@ extern "C" kvm_status kvm_update_round(kvm_ctx* c, const kvm_round* r, void* str
     return KVM_OK;
 }
 
+namespace {
+// The canary bands of every buffer, read back (debug builds; a no-op otherwise).
+kvm_status check_canaries(kvm_ctx* c) {
+    if (!kCanary) return KVM_OK;
+    std::vector<unsigned char> band(kCanary);
+    for (const auto& a : c->allocs) {
+        for (int side = 0; side < 2; ++side) {
+            const char* src = static_cast<const char*>(a.base) + (side ? kCanary + a.bytes : 0);
+            CUDA_TRY(cudaMemcpy(band.data(), src, kCanary, cudaMemcpyDeviceToHost));
+            for (size_t i = 0; i < kCanary; ++i)
+                if (band[i] != kCanaryByte)
+                    return fail(KVM_E_DEVICE, "canary band %s buffer %s overwritten (byte %zu)",
+                                side ? "after" : "before", a.name, i);
+        }
+    }
+    return KVM_OK;
+}
+}  // namespace
+
+extern "C" kvm_status kvm_debug_poke_canary(kvm_ctx* c) {
+    if (!c) return fail(KVM_E_INVAL, "NULL context");
+    if (!kCanary) return fail(KVM_E_UNSUPPORTED, "canary bands exist only in builds with -DKVM_DEBUG");
+    if (c->allocs.empty()) return fail(KVM_E_INVAL, "the context owns no device buffer");
+    const auto& a = c->allocs.front();
+    CUDA_TRY(cudaDeviceSynchronize());
+    CUDA_TRY(cudaMemset(static_cast<char*>(a.base) + kCanary + a.bytes, 0, 1));   // first byte past the buffer
+    return KVM_OK;
+}
+
 extern "C" kvm_status kvm_check(kvm_ctx* c, void* stream) {
     if (!c) return fail(KVM_E_INVAL, "NULL context");
     CUDA_TRY(cudaStreamSynchronize((cudaStream_t)stream));
+    {
+        const kvm_status cs = check_canaries(c);
+        if (cs) return cs;
+    }
     int32_t e = 0;
     CUDA_TRY(cudaMemcpy(&e, c->err, 4, cudaMemcpyDeviceToHost));
     if (e) {

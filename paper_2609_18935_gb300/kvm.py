@@ -98,6 +98,7 @@ _SIGS = {
                                          C.POINTER(C.c_int32), C.c_void_p]),
     "kvm_kv_compact_noalloc_check": (C.c_int, [C.c_void_p]),
     "kvm_debug_compact_wait": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
+    "kvm_debug_poke_canary": (C.c_int, [C.c_void_p]),
     "kvm_attn_probe": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                  C.c_int32, C.c_void_p, C.c_void_p]),
     "kvm_effective_group_count": (C.c_int, [C.c_int32, C.POINTER(C.c_double), C.POINTER(C.c_double)]),
@@ -501,6 +502,10 @@ class Context:
         failure-detection stall (every later compaction block waits on a word
         nothing sets and gives up after `polls` polls)."""
         _check(_lib.kvm_debug_compact_wait(self._h, int(polls), int(bool(stall))))
+
+    def debug_poke_canary(self):
+        """kvm_debug_poke_canary (debug builds): spoil one canary byte."""
+        _check(_lib.kvm_debug_poke_canary(self._h))
 
     def launch_count(self) -> int:
         return int(_lib.kvm_launch_count(self._h))

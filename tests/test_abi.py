@@ -87,3 +87,13 @@ def test_null_context_is_rejected(lib):
     assert lib.kvm_advance(None, None) == kvm.KVM_E_INVAL
     assert lib.kvm_check(None, None) == kvm.KVM_E_INVAL
     assert lib.kvm_launch_count(None) == 0
+
+
+def test_debug_build_exports_the_same_symbols():
+    """The canary-checking build (-DKVM_DEBUG) compiles and exports the same
+    C ABI as the release library."""
+    from paper_2609_18935_gb300 import build_lib
+    path = build_lib.build(debug=True)
+    out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (kvm_\w+)$", out, flags=re.M))
+    assert set(_declared()) <= exported
