@@ -452,6 +452,17 @@ kvm_status kvm_profile_read(kvm_ctx* ctx, int32_t kernel, int64_t* launches, dou
  * check. */
 kvm_status kvm_check(kvm_ctx* ctx, void* stream);
 
+/* Launch plans (no paper counterpart; the results are bit-identical either
+ * way).  what = KVM_FUSE_GDN, enable != 0 (the default): when a round has
+ * few characters and long tails, each delta-rule layer runs as one launch
+ * in which some blocks scan the chunks in order while the others prepare
+ * later chunks' records (published through flags in the context's
+ * workspace); enable = 0: a prep launch, then a scan launch.  If the device
+ * refuses the one-launch form, the context uses two launches from then on.
+ * Errors: KVM_E_INVAL. */
+enum { KVM_FUSE_GDN = 0 };
+kvm_status kvm_set_fusion(kvm_ctx* ctx, int32_t what, int32_t enable);
+
 /* Failure-detection hook of the compaction's bounded waits (no paper
  * counterpart).  polls: how many times a compaction block polls an earlier
  * chunk's read flag before it gives up (0 restores the default, ~0.3-1 s).

@@ -18,8 +18,9 @@
 // it leaves per (chunk, head) a record with [W; Q'] and K as ready-made MMA
 // operand images, U and A U in fp32, w and G_C.  The scan kernel then walks
 // the chunks of each (character, head, d_v slice) in order with the state in
-// TMEM: one bulk copy of the next record's images (double-buffered), the MMA
-// [W; Q'] S0^T, E and O, and the state update.
+// TMEM: each of the next record's images is fetched by one bulk copy as soon
+// as the current one has been consumed; the MMA [W; Q'] S0^T, E and O, and
+// the state update follow, with four block barriers per chunk.
 //
 // Tensor-core operands are bf16.  K, Q, V are exact in bf16 and used in place
 // (K and V as MN-major operands in their natural row layout).  Every computed
@@ -124,8 +125,83 @@ struct PrepCfg {
     static constexpr uint32_t T_WU = 128;                    // [W | U] (DK + dv cols)
 };
 
+// Fused launches (gdn_fused_kernel): a finished record is published by
+// setting its flag to the launch's epoch; the scan waits for it.  Standalone
+// launches pass flags = null (the records complete with the prep grid).
+struct FuseCtl {
+    uint32_t* flags;      // [record][kFlagWords], record = chunk * H + head
+    uint32_t epoch;
+};
+constexpr int kFlagWords = 32;   // one flag per 128-byte line
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release_u32(uint32_t* p, uint32_t v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Orders this thread's async-proxy (bulk copy) accesses of global memory
+// with its generic-proxy ones.
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// Record `rec` (chunk * H + head) of a fused launch: wait (one thread,
+// bounded in wall time) until the prep has published it, then order the
+// bulk copies that follow after that observation.
+__device__ __forceinline__ bool wait_record(const FuseCtl& fc, int64_t rec, volatile int* abort_flag, int* err,
+                                            int* diag, int tag) {
+    if (!fc.flags) return true;
+    const uint32_t* f = fc.flags + rec * kFlagWords;
+    uint64_t t0 = 0;
+    for (uint32_t it = 0;; ++it) {
+        if (ld_acquire_u32(f) == fc.epoch) {
+            fence_proxy_async_global();
+            return true;
+        }
+        if ((it & 15) == 15) {
+            if (*abort_flag) return false;
+            const uint64_t now = globaltimer_ns();
+            if (t0 == 0) t0 = now;
+            else if (now - t0 > 250000000ull) {
+                *abort_flag = 1;
+                atomicOr(err, kErrWait);
+                if (diag && atomicCAS(diag, 0, (int)blockIdx.x + 1) == 0) {
+                    diag[1] = tag;
+                    diag[2] = 0;
+                }
+                return false;
+            }
+        }
+        __nanosleep(32);
+    }
+}
+
+// Work unit u of a fused launch's prep workers: units are ordered by the
+// chunk's index within its character, then character, then head, so that
+// every character's scan finds its next chunk ready early.  Returns
+// chunk * H + head, or -1 past the last unit.
+__device__ __forceinline__ int fused_unit(const GdnParams& p, int u) {
+    for (int i = 0;; ++i) {
+        bool any = false;
+        for (int b = 0; b < p.n_chars; ++b) {
+            if ((p.ch[b].M + C - 1) / C > i) {
+                if (u < p.H) return (p.ch[b].chunk_off + i) * p.H + u;
+                u -= p.H;
+                any = true;
+            }
+        }
+        if (!any) return -1;
+    }
+}
+
+// The prep's work units u = u0, u0 + ustride, ... (standalone: one unit per
+// block, u = blockIdx.x over (chunk, head, part); fused: the units of
+// fused_unit, one part each).
 template <int DK>
-__global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_constant__ GdnParams p) {
+__device__ __forceinline__ void gdn_prep_run(const GdnParams& p, const FuseCtl& fc, int u0, int ustride) {
     using G = PrepCfg<DK>;
     using R = Rec<DK>;
     extern __shared__ uint8_t smem_raw[];
@@ -146,20 +222,8 @@ __global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_
     const int row = q4 * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     const int H = p.H, dv = p.dv;
-    // with two parts per (chunk, head) both solve for X; part 0 writes the
-    // [W; Q'] and K images, part 1 U | A U and w, G_C
-    const int part = blockIdx.x % p.prep_parts;
-    const int ch_h = blockIdx.x / p.prep_parts;
-    const bool do_w = p.prep_parts == 1 || part == 0;
-    const bool do_u = p.prep_parts == 1 || part == 1;
-    const int chunk = ch_h / H, h = ch_h % H;
-    const int b = find_char_by_chunk(p, chunk);
-    const GdnChar ch = p.ch[b];
-    const int c0 = (chunk - ch.chunk_off) * C;
-    if (c0 >= ch.M) return;                          // uniform per block (not reached for valid grids)
-    const int n = min(C, ch.M - c0);
-    const int64_t tok0 = ch.tail_off + c0;
-    uint8_t* rec = p.work + ((int64_t)chunk * H + h) * p.rec_bytes;
+    const int parts = fc.flags ? 1 : p.prep_parts;
+    const int n_units = p.total_chunks * H * parts;
 
     if (tid == 0) {
         abort_flag = 0;
@@ -170,8 +234,27 @@ __global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_
         tmem_alloc(smem_u32(tmem_slot), 512);
         tmem_relinquish();
     }
-    grid_dependency_wait();
-    grid_dependents_launch();
+    if (!fc.flags) {                                 // the fused kernel waited already
+        grid_dependency_wait();
+        grid_dependents_launch();
+    }
+    uint32_t phase = 0;
+    for (int u = u0; u < n_units; u += ustride) {
+    // with two parts per (chunk, head) both solve for X; part 0 writes the
+    // [W; Q'] and K images, part 1 U | A U and w, G_C
+    const int part = u % parts;
+    const int ch_h = fc.flags ? fused_unit(p, u) : u / parts;
+    if (ch_h < 0) break;                             // uniform per block (not reached for valid grids)
+    const bool do_w = parts == 1 || part == 0;
+    const bool do_u = parts == 1 || part == 1;
+    const int chunk = ch_h / H, h = ch_h % H;
+    const int b = find_char_by_chunk(p, chunk);
+    const GdnChar ch = p.ch[b];
+    const int c0 = (chunk - ch.chunk_off) * C;
+    if (c0 >= ch.M) continue;                        // uniform per block (not reached for valid grids)
+    const int n = min(C, ch.M - c0);
+    const int64_t tok0 = ch.tail_off + c0;
+    uint8_t* rec = p.work + ((int64_t)chunk * H + h) * p.rec_bytes;
     // ---- loads (every global load issued before the shared stores)
     {
         constexpr int NKQ = 128 * (DK / 8) / kPrepThreads;
@@ -236,9 +319,9 @@ __global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_
             float* misc = reinterpret_cast<float*>(rec + R::misc_off(dv));
             misc[tid] = tid < n ? bs[tid] * expf(gs[n - 1] - gs[tid]) : 0.f;     // w_j
             if (tid == 0) misc[C] = expf(gs[n - 1]);                            // G_C
+            if (fc.flags) __threadfence();                                      // before the record's flag
         }
     }
-    uint32_t phase = 0;
     bool ok = true;
     // the issuing thread waits for its MMAs and the block follows it at the
     // barrier (waiting lanes of the issuer's warp would slow its issue)
@@ -534,17 +617,34 @@ __global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_
         }
         if (tid == 0) {
             // the sources must be read before the block's shared memory is
-            // released; the writes complete with the grid, before the scan
-            // (which waits on this grid) reads them
+            // released or restaged; standalone, the writes complete with the
+            // grid, before the scan (which waits on this grid) reads them
             bulk_wait_read();
         }
     }
     tc_fence_before();
+    __syncthreads();                                 // the staging area is free for the next unit
+    tc_fence_after();
+    if (fc.flags && tid == 0 && ok) {
+        // fused: publish the record once its writes have completed (the
+        // other threads are already loading the next unit)
+        bulk_wait_all();
+        fence_proxy_async_global();
+        __threadfence();
+        st_release_u32(fc.flags + (int64_t)ch_h * kFlagWords, fc.epoch);
+    }
+    }  // units
+    tc_fence_before();
     __syncthreads();
     if (warp == 0) {
         tc_fence_after();
-        tmem_dealloc(tmem, 512);
+        tmem_dealloc(*tmem_slot, 512);
     }
+}
+
+template <int DK>
+__global__ void __launch_bounds__(kPrepThreads, 1) gdn_prep_kernel(const __grid_constant__ GdnParams p) {
+    gdn_prep_run<DK>(p, FuseCtl{nullptr, 0}, blockIdx.x, gridDim.x);
 }
 
 // ============================================================================
@@ -568,8 +668,12 @@ struct ScanCfg {
 
 // CW: columns of the slice a thread handles per TMEM access (16 when the
 // slice is 32 wide, so that all eight warps share the elementwise phases)
+// One scan item: character b, head h, d_v rows r0 .. r0 + dv_slice - 1.
+// Written for 256 threads (eight warps: lane quarter x column half); in a
+// fused launch's 512-thread blocks the other eight warps only take part in
+// the block barriers (their column range is empty).
 template <int DK, int CW>
-__global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_constant__ GdnParams p) {
+__device__ __forceinline__ void gdn_scan_run(const GdnParams& p, const FuseCtl& fc, int b, int h, int r0) {
     using G = ScanCfg<DK>;
     using R = Rec<DK>;
     extern __shared__ uint8_t smem_raw[];
@@ -591,9 +695,6 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     const int row = q4 * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     const int dvs = p.dv_slice;
-    const int r0 = blockIdx.x * dvs;
-    const int h = blockIdx.y;
-    const int b = blockIdx.z;
     const GdnChar ch = p.ch[b];
     if (ch.M <= 0) return;                           // uniform per block; touches no memory
     const int H = p.H, dv = p.dv;
@@ -652,9 +753,13 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     // The state slice comes from an earlier round (or kvm_set_state), which
     // completed before the prep kernel this launch follows had started, so
     // it is staged before waiting for that kernel; its records are not.
-    grid_dependency_wait();
-    grid_dependents_launch();
-    if (tid == 0) {
+    if (!fc.flags) {                                 // the fused kernel waited already
+        grid_dependency_wait();
+        grid_dependents_launch();
+    }
+    // fused: the first record must have been published (a failed wait
+    // raises the abort flag, which stops the block at its first MMA wait)
+    if (tid == 0 && wait_record(fc, (int64_t)ch.chunk_off * H + h, &abort_flag, p.err, p.diag, 0x5f)) {
         mbar_arrive_expect_tx(bar_wq, G::WQ);
         bulk_load(sb + G::OFF_WQ, rec_of(0), G::WQ, bar_wq);
         mbar_arrive_expect_tx(bar_k, G::KI);
@@ -686,13 +791,16 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         const int64_t tok0 = ch.tail_off + (int64_t)i * C;
         const uint8_t* rec = rec_of(i);
         const float* misc = reinterpret_cast<const float*>(rec + R::misc_off(dv));
-        const float wt = __ldg(misc + (row & 63));
-        const float gC = __ldg(misc + C);
-        ok = mbar_wait(bar_wq, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x51 + 256 * i);
-        ok = __syncthreads_and(ok);
-        if (!ok) break;
+        // L2-coherent loads: in a fused launch the record was written by
+        // another block of this grid
+        const float wt = __ldcg(misc + (row & 63));
+        const float gC = __ldcg(misc + C);
         // ---------------------------------------------------------------- [W; Q'] S0^T
-        if (tid == 0) {
+        // Only the issuing thread reads the [W; Q'] image, so only it waits
+        // for the copy; the state operand was published by the barrier that
+        // ended the previous chunk.  A failed wait raises the abort flag,
+        // which the MMA wait below turns into a block-wide stop.
+        if (tid == 0 && mbar_wait(bar_wq, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x51 + 256 * i)) {
             tc_fence_after();
 #pragma unroll
             for (int ks = 0; ks < DK / 16; ++ks) {
@@ -710,13 +818,17 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         }
         ok = mma_wait();
         if (!ok) break;
-        if (tid == 0 && i + 1 < nch) {               // [W;Q'] image consumed: fetch the next one
+        // [W;Q'] image consumed: fetch the next one (fused: once the prep
+        // has published that record; a failed wait raises the abort flag)
+        if (tid == 0 && i + 1 < nch &&
+            wait_record(fc, (int64_t)(ch.chunk_off + i + 1) * H + h, &abort_flag, p.err, p.diag, 0x5e + 256 * i)) {
             mbar_arrive_expect_tx(bar_wq, G::WQ);
             bulk_load(sb + G::OFF_WQ, rec_of(i + 1), G::WQ, bar_wq);
         }
-        ok = __syncthreads_and(mbar_wait(bar_u, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x52 + 256 * i));
-        if (!ok) break;
         // ---------------------------------------------------------------- E, O; S^T *= G_C
+        // every thread waits for the U | A U copy it reads; a failed wait
+        // stops the block at the barrier after this phase
+        const bool u_ok = mbar_wait(bar_u, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x52 + 256 * i);
         {
             const int t = row & 63;
 #pragma unroll
@@ -768,15 +880,17 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
             }
             tmem_st_wait();
         }
-        issue_begin();
-        if (tid == 0 && i + 1 < nch) {               // U | A U consumed: fetch the next one
+        fence_proxy_async_smem();
+        tc_fence_before();
+        ok = __syncthreads_and(u_ok);
+        if (!ok) break;
+        if (tid == 0 && i + 1 < nch && !abort_flag) {   // U | A U consumed: fetch the next one
             mbar_arrive_expect_tx(bar_u, ubytes);
             bulk_load(sb + G::OFF_U, rec_of(i + 1) + uslice, ubytes, bar_u);
         }
         // ---------------------------------------------------------------- S^T += K^T (w E)
-        ok = __syncthreads_and(mbar_wait(bar_k, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x53 + 256 * i));
-        if (!ok) break;
-        if (tid == 0) {
+        // only the issuing thread reads the K image
+        if (tid == 0 && mbar_wait(bar_k, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x53 + 256 * i)) {
             tc_fence_after();
 #pragma unroll
             for (int ks = 0; ks < C / 16; ++ks) {
@@ -788,7 +902,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
         }
         ok = mma_wait();
         if (!ok) break;
-        if (tid == 0 && i + 1 < nch) {               // K image consumed: fetch the next one
+        if (tid == 0 && i + 1 < nch && !abort_flag) {   // K image consumed: fetch the next one
             mbar_arrive_expect_tx(bar_k, G::KI);
             bulk_load(sb + G::OFF_K, rec_of(i + 1) + G::WQ, G::KI, bar_k);
         }
@@ -840,6 +954,35 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
     }
 }
 
+template <int DK, int CW>
+__global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_constant__ GdnParams p) {
+    gdn_scan_run<DK, CW>(p, FuseCtl{nullptr, 0}, blockIdx.z, blockIdx.y, blockIdx.x * p.dv_slice);
+}
+
+// ============================================================================
+// fused: prep and scan in one launch.  Blocks 0 .. n_scan-1 each run one scan
+// item (character, head, d_v slice); the others are prep workers that take
+// the (chunk, head) units in fused_unit order and publish each record through
+// its flag.  A scan waits only for records, and prep workers never wait, so
+// the launch completes as long as all of its blocks can be resident at once:
+// the grid is at most one block per SM (launched cooperatively), and the
+// kernels after it on the stream cannot take an SM before every block of it
+// has started (their launch waits for every block's launch_dependents).
+// ============================================================================
+template <int DK, int CW>
+__global__ void __launch_bounds__(kPrepThreads, 1) gdn_fused_kernel(const __grid_constant__ GdnParams p) {
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const FuseCtl fc{p.flags, p.epoch};
+    const int x = blockIdx.x;
+    if (x < p.n_scan) {
+        const int slices = p.dv / p.dv_slice;
+        gdn_scan_run<DK, CW>(p, fc, x / (slices * p.H), (x / slices) % p.H, (x % slices) * p.dv_slice);
+    } else {
+        gdn_prep_run<DK>(p, fc, x - p.n_scan, gridDim.x - p.n_scan);
+    }
+}
+
 // Opt in to the kernel's dynamic shared memory once per device (one flag per
 // kernel: the template is keyed on the kernel itself).
 template <auto KERNEL>
@@ -872,6 +1015,25 @@ void launch_scan_dk(const GdnParams& p, cudaStream_t s) {
     else launch_scan_cw<DK, 32>(p, s);
 }
 
+template <int DK>
+cudaError_t launch_fused_dk(const GdnParams& p, int grid, cudaStream_t s) {
+    constexpr int smem = ScanCfg<DK>::SMEM > PrepCfg<DK>::SMEM ? ScanCfg<DK>::SMEM : PrepCfg<DK>::SMEM;
+    configure_once<gdn_fused_kernel<DK, 16>>(smem);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kPrepThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeCooperative;             // every block resident at once
+    at[0].val.cooperative = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, gdn_fused_kernel<DK, 16>, p);
+}
+
 }  // namespace
 
 int64_t gdn_record_bytes(int dk, int dv) {
@@ -882,6 +1044,12 @@ void launch_gdn_chunk_prep(const GdnParams& p, cudaStream_t s) {
     if (p.total_chunks <= 0) return;
     if (p.dk == 64) launch_prep_dk<64>(p, s);
     else if (p.dk == 128) launch_prep_dk<128>(p, s);
+}
+
+cudaError_t launch_gdn_fused(const GdnParams& p, int grid, cudaStream_t s) {
+    if (p.total_chunks <= 0) return cudaSuccess;
+    if (p.dv_slice > 32) return cudaErrorInvalidValue;    // the 512-thread blocks leave 128 registers a thread
+    return p.dk == 64 ? launch_fused_dk<64>(p, grid, s) : launch_fused_dk<128>(p, grid, s);
 }
 
 void launch_gdn_chunk_scan(const GdnParams& p, cudaStream_t s) {

@@ -229,6 +229,11 @@ struct GdnParams {
     int32_t total_chunks;     // sum over characters of ceil(M / 64)
     int32_t* err;
     int32_t* diag;            // first expired wait: block + 1, tag, parity
+    // fused launches (launch_gdn_fused): the first n_scan blocks are scan
+    // items, the rest prep workers; record r is published by flags[32 r] = epoch
+    int32_t n_scan;
+    uint32_t epoch;
+    uint32_t* flags;
     GdnChar ch[kMaxChars];
 };
 
@@ -255,6 +260,9 @@ void launch_gdn_conv(const ConvParams& p, cudaStream_t s);
 int64_t gdn_record_bytes(int dk, int dv);
 void launch_gdn_chunk_prep(const GdnParams& p, cudaStream_t s);   // state-independent chunk products
 void launch_gdn_chunk_scan(const GdnParams& p, cudaStream_t s);   // chunks in order, state in TMEM
+// Both in one launch of `grid` blocks (one per SM at most); returns the
+// launch's error (the caller falls back to the two launches).
+cudaError_t launch_gdn_fused(const GdnParams& p, int grid, cudaStream_t s);
 
 // Set the text returned by kvm_last_error() and return `code`.
 int report_error(int code, const char* msg);

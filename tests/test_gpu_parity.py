@@ -261,3 +261,35 @@ def test_host_resident_round_equals_device_round(arena):
                         vd.view(torch.int16), vh.view(torch.int16)), (r, l, b)
         live = [dev.get_live(b)[0] for b in range(2)]
         assert live == [host.get_live(b)[0] for b in range(2)]
+
+
+@pytest.mark.parametrize("n_chars,tails", [(1, [256]), (1, [1024]), (2, [130, 64]), (1, [1])])
+def test_delta_rule_launch_plans_agree(n_chars, tails):
+    """The delta-rule layer as one launch (prep workers publishing records
+    to scan blocks in the same grid) and as a prep launch followed by a scan
+    launch run the same arithmetic: outputs and states bit-identical, over
+    two rounds."""
+    import torch
+    from paper_2609_18935_gb300 import kvm
+    shape = W.ModelShape([W.GDN, W.GDN], 16, 2, 256, 64, 1e4, 16, 128, 128)
+    mk = lambda: kvm.Context(shape.layer_kind, 16, 2, 256, 64, 1e4, 16, 128, 128, [2 * max(tails) + 64] * n_chars,
+                             sum(tails))
+    a, b = mk(), mk()
+    b.set_gdn_fusion(False)
+    w = W.Workload("plans", 55, shape, [0] * n_chars, 2)
+    for ctx in (a, b):
+        for l in (0, 1):
+            ctx.set_state(l, torch.from_numpy(np.stack([W.prefix_state(w, c, l) for c in range(n_chars)])).cuda())
+    tail_cu = np.concatenate([[0], np.cumsum(tails)]).astype(np.int32)
+    z = np.zeros(n_chars + 1, np.int32)
+    for r in range(2):
+        ins = W.device_round_inputs(w, 900 + r, tails)
+        outs = [{l: torch.empty((sum(tails), 16, 128), dtype=torch.bfloat16, device="cuda") for l in (0, 1)}
+                for _ in range(2)]
+        a.update_round(z, [], [], tail_cu, ins, outs[0])
+        b.update_round(z, [], [], tail_cu, ins, outs[1])
+        a.check()
+        b.check()
+        for l in (0, 1):
+            assert torch.equal(outs[0][l].view(torch.int16), outs[1][l].view(torch.int16)), (r, l)
+            assert torch.equal(a.get_state(l), b.get_state(l)), (r, l)
