@@ -367,9 +367,9 @@ kvm_status kvm_update_round(kvm_ctx* ctx, const kvm_round* round, void* stream);
  * inside the library (every GPU that loads the library holds it until the
  * process exits); this call allocates nothing.  Limits: n_slabs <= 512,
  * n_spans <= 1024, head_dim in {64, 128, 256}, and
- * 2 * n_slabs * ceil(moved / (8192 / head_dim)) + ceil(moved / 1024) <= 65536
+ * 2 * n_slabs * ceil(moved / (16384 / head_dim)) + ceil(moved / 2048) <= 65536
  * where moved = rows from the first span to the new live end (e.g. 24 slabs
- * of head_dim 256 allow ~43K moved rows); larger requests return
+ * of head_dim 256 allow ~87K moved rows); larger requests return
  * KVM_E_CAPACITY.  The first call on each device looks up the array's device
  * address (cudaGetSymbolAddress); make that first call before any stream
  * capture.  Every call shares the one array and clears the part it uses, so

@@ -46,7 +46,7 @@ constexpr int kErrWait = 2;         // a bounded wait expired
 // kv_compact
 // ----------------------------------------------------------------------------
 constexpr int kCompactThreads = 256;
-constexpr int kCompactVecPerThread = 4;            // 16-byte vectors held per thread
+constexpr int kCompactVecPerThread = 8;            // 16-byte vectors held per thread (8: 418 us against 531 with 4 for the 1.5 GB of the 48-layer round)
 constexpr int kCompactVecPerChunk = kCompactThreads * kCompactVecPerThread;
 constexpr int kCompactWaitLimit = 1 << 22;        // default polls of a read flag (~0.3-1 s with the back-off)
 
