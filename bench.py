@@ -317,12 +317,15 @@ def job_throughput(world: int, tokens_per_rank: float, ms: float) -> float:
 
 def workload_config(w, args, world):
     s = w.shape
-    full = W.make_workload(args.workload)
+    full = W.make_workload(args.workload, args.layers)
     if world > 1 and full.n_chars > 1:
         par = f"population of {full.n_chars} characters partitioned over {world} ranks (balanced by M L')"
     else:
         par = f"{world} independent replica(s), characters per rank fixed"
-    return {"workload": WORKLOAD_TEXT[args.workload], "name": args.workload, "chars": full.n_chars,
+    text = WORKLOAD_TEXT[args.workload]
+    if args.layers:
+        text += f" (shortened to {len(s.layer_kind)} layers for a profiling capture)"
+    return {"workload": text, "name": args.workload, "chars": full.n_chars,
             "layers": len(s.layer_kind), "chain_rounds": w.rounds,
             "l2": "flushed before every step (256 MiB write), outside the timed events",
             "parallelism": par}
@@ -332,7 +335,7 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    w = W.make_workload(args.workload)
+    w = W.make_workload(args.workload, args.layers)
     m = REFERENCE_TOKENS[args.workload]
     st = oracle_state(w)
     for _ in range(args.warmup):
@@ -409,7 +412,7 @@ def run_kvm(args):
             dist.barrier()
     kvm.load_library()
 
-    w, scaling = rank_share(W.make_workload(args.workload), rank, world)
+    w, scaling = rank_share(W.make_workload(args.workload, args.layers), rank, world)
     s = w.shape
     plan = W.simulate_plan(w)
     R = len(plan)
@@ -646,6 +649,9 @@ def main():
     ap.add_argument("--impl", choices=["kvm", "reference"], default="kvm")
     ap.add_argument("--workload", choices=list(WORKLOAD_TEXT), default="long")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="shorter stack of the same 3:1 pattern and shapes (profiling captures that must hold "
+                         "a few GB on the device); the default is the workload's own stack")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -452,16 +452,26 @@ kvm_status kvm_profile_read(kvm_ctx* ctx, int32_t kernel, int64_t* launches, dou
  * check. */
 kvm_status kvm_check(kvm_ctx* ctx, void* stream);
 
-/* Launch plans (no paper counterpart; the results are bit-identical either
- * way).  what = KVM_FUSE_GDN, enable != 0 (the default): when a round has
- * few characters and long tails, each delta-rule layer runs as one launch
- * in which some blocks scan the chunks in order while the others prepare
- * later chunks' records (published through flags in the context's
- * workspace); enable = 0: a prep launch, then a scan launch.  If the device
- * refuses the one-launch form, the context uses two launches from then on.
+/* Launch plans of the delta-rule layers (no paper counterpart; fused
+ * defaults to on, state chain to off).
+ * KVM_PLAN_GDN_STATE_CHAIN (d_k = d_v = 128, one or few characters): the
+ * serial chunk chain carries only the state, S^T <- P_c S^T + B_c with
+ * P_c = G_C I - K^T diag(w) W and B_c = K^T diag(w) U formed in the
+ * parallel prep, and the chunks' outputs O = A U + Q' S0^T follow in one
+ * parallel pass over per-chunk state snapshots.  Off: the chain also forms
+ * E = U - W S0^T and the outputs.  The two forms round differently (both
+ * within the library's accuracy).  Measured in a stack of delta-rule layers
+ * (1024-token tail): the state chain takes 36 us against 52 for the full
+ * chain, but its larger prep and the output pass make a layer 86 us against
+ * 60, so it is off by default.
+ * KVM_PLAN_GDN_FUSED: when a round has few characters and long tails, the
+ * prep and the chain run in one launch, prep blocks publishing each chunk's
+ * record through flags to the chain blocks; off: a prep launch, then the
+ * chain's.  Bit-identical either way.  If the device refuses the one-launch
+ * form, the context uses two launches from then on.
  * Errors: KVM_E_INVAL. */
-enum { KVM_FUSE_GDN = 0 };
-kvm_status kvm_set_fusion(kvm_ctx* ctx, int32_t what, int32_t enable);
+enum { KVM_PLAN_GDN_FUSED = 0, KVM_PLAN_GDN_STATE_CHAIN = 1 };
+kvm_status kvm_set_plan(kvm_ctx* ctx, int32_t what, int32_t enable);
 
 /* Failure-detection hook of the compaction's bounded waits (no paper
  * counterpart).  polls: how many times a compaction block polls an earlier

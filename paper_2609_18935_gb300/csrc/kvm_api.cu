@@ -123,6 +123,10 @@ struct kvm_ctx {
     uint32_t* gdn_flags = nullptr;
     uint32_t gdn_epoch = 0;
     bool gdn_fuse = true;
+    // state-chain form (d_k = d_v = 128): per-chunk snapshots of the state
+    uint8_t* gdn_snap = nullptr;
+    int64_t gdn_snap_bytes = 0;
+    bool gdn_chain = false;
     // staging for host-resident rounds: every layer's inputs (q, k, v, alpha,
     // beta) and output have their own buffers, so the copies of all layers
     // run on a copy stream beside the kernels
@@ -515,6 +519,10 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         const size_t chunks = (size_t)max_tail_tokens / 64 + n_chars;
         if (e == cudaSuccess) e = alloc_dev(c, &c->gdn_work, chunks * c->H * c->gdn_rec, "gdn_work", false);
         if (e == cudaSuccess) e = alloc_dev(c, &c->gdn_flags, chunks * c->H * 32, "gdn_flags");
+        if (c->dk == 128 && c->dv == 128) {
+            c->gdn_snap_bytes = gdn_snapshot_bytes(c->dk, c->dv);
+            if (e == cudaSuccess) e = alloc_dev(c, &c->gdn_snap, chunks * c->H * c->gdn_snap_bytes, "gdn_snap", false);
+        }
     }
     {
         size_t total_stage = 0;
@@ -1153,7 +1161,32 @@ kvm_status do_gdn(kvm_ctx* c, int layer, const int32_t* tail_cu, const void* q, 
     // prep is a single wave either way.  Otherwise the prep grid, then the scan.
     const int items = c->B * c->H * (c->dv / p.dv_slice);
     const int workers = c->num_sms - items;
-    if (c->gdn_fuse && p.dv_slice <= 32 && workers >= kMinPrepWorkers && chunks * c->H >= 2 * workers) {
+    const bool fuse = c->gdn_fuse && p.dv_slice <= 32 && workers >= kMinPrepWorkers && chunks * c->H >= 2 * workers;
+    if (c->gdn_chain && c->gdn_snap && p.dv_slice == 32) {
+        // state-chain form: the chain carries only S (one MMA batch a chunk),
+        // the outputs follow in a parallel pass over per-chunk snapshots
+        p.snap = c->gdn_snap;
+        p.snap_bytes = c->gdn_snap_bytes;
+        p.n_scan = items;
+        p.flags = c->gdn_flags;
+        if (fuse) p.epoch = ++c->gdn_epoch;
+        const int ps = prof_begin(c, KVM_K_GDN, s);
+        const cudaError_t e = launch_gdn_v2(p, fuse ? std::min(c->num_sms, items + chunks * c->H) : 0, s);
+        prof_end(c, ps, s);
+        if (e == cudaSuccess) {
+            LAUNCH_CHECK(c);
+            return KVM_OK;
+        }
+        (void)cudaGetLastError();                     // the fused launch was refused: two launches from now on
+        c->gdn_fuse = false;
+        const int ps2 = prof_begin(c, KVM_K_GDN, s);
+        const cudaError_t e2 = launch_gdn_v2(p, 0, s);
+        prof_end(c, ps2, s);
+        if (e2 != cudaSuccess) return fail(KVM_E_CUDA, "delta-rule launch failed: %s", cudaGetErrorString(e2));
+        LAUNCH_CHECK(c);
+        return KVM_OK;
+    }
+    if (fuse) {
         p.n_scan = items;
         p.epoch = ++c->gdn_epoch;
         p.flags = c->gdn_flags;
@@ -1627,11 +1660,12 @@ extern "C" kvm_status kvm_check(kvm_ctx* c, void* stream) {
     return KVM_OK;
 }
 
-extern "C" kvm_status kvm_set_fusion(kvm_ctx* c, int32_t what, int32_t enable) {
+extern "C" kvm_status kvm_set_plan(kvm_ctx* c, int32_t what, int32_t enable) {
     if (!c) return fail(KVM_E_INVAL, "NULL context");
     switch (what) {
-        case KVM_FUSE_GDN: c->gdn_fuse = enable != 0; break;
-        default: return fail(KVM_E_INVAL, "unknown fusion %d", what);
+        case KVM_PLAN_GDN_FUSED: c->gdn_fuse = enable != 0; break;
+        case KVM_PLAN_GDN_STATE_CHAIN: c->gdn_chain = enable != 0; break;
+        default: return fail(KVM_E_INVAL, "unknown plan option %d", what);
     }
     return KVM_OK;
 }

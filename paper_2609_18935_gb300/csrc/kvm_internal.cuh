@@ -234,6 +234,9 @@ struct GdnParams {
     int32_t n_scan;
     uint32_t epoch;
     uint32_t* flags;
+    // v2: the state entering each chunk, per (chunk, head), as the output pass reads it
+    uint8_t* snap;
+    int64_t snap_bytes;
     GdnChar ch[kMaxChars];
 };
 
@@ -263,6 +266,11 @@ void launch_gdn_chunk_scan(const GdnParams& p, cudaStream_t s);   // chunks in o
 // Both in one launch of `grid` blocks (one per SM at most); returns the
 // launch's error (the caller falls back to the two launches).
 cudaError_t launch_gdn_fused(const GdnParams& p, int grid, cudaStream_t s);
+// v2 (d_k = 128, 32-row slices): prep, state chain and output pass (or, with
+// fused_grid > 0, prep and chain in one launch of fused_grid blocks, then the
+// output pass).  Returns a refused launch's error before enqueuing anything else.
+int64_t gdn_snapshot_bytes(int dk, int dv);
+cudaError_t launch_gdn_v2(const GdnParams& p, int fused_grid, cudaStream_t s);
 
 // Set the text returned by kvm_last_error() and return `code`.
 int report_error(int code, const char* msg);

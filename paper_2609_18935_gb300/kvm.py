@@ -18,7 +18,7 @@ LIB_PATH = os.environ.get("KVM_LIB", os.path.join(_PKG, "_build", "libkvm.so"))
 
 KVM_OK, KVM_E_INVAL, KVM_E_SPAN, KVM_E_CAPACITY, KVM_E_CUDA, KVM_E_DEVICE, KVM_E_UNSUPPORTED = range(7)
 LAYER_GDN, LAYER_ATTN = 0, 1
-FUSE_GDN = 0
+PLAN_GDN_FUSED, PLAN_GDN_STATE_CHAIN = 0, 1
 
 _ERRNAMES = {1: "KVM_E_INVAL", 2: "KVM_E_SPAN", 3: "KVM_E_CAPACITY", 4: "KVM_E_CUDA",
              5: "KVM_E_DEVICE", 6: "KVM_E_UNSUPPORTED"}
@@ -100,7 +100,7 @@ _SIGS = {
     "kvm_kv_compact_noalloc_check": (C.c_int, [C.c_void_p]),
     "kvm_debug_compact_wait": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
     "kvm_debug_poke_canary": (C.c_int, [C.c_void_p]),
-    "kvm_set_fusion": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
+    "kvm_set_plan": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32]),
     "kvm_attn_probe": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                  C.c_int32, C.c_void_p, C.c_void_p]),
     "kvm_effective_group_count": (C.c_int, [C.c_int32, C.POINTER(C.c_double), C.POINTER(C.c_double)]),
@@ -506,9 +506,14 @@ class Context:
         _check(_lib.kvm_debug_compact_wait(self._h, int(polls), int(bool(stall))))
 
     def set_gdn_fusion(self, enable=True):
-        """kvm_set_fusion(KVM_FUSE_GDN): one launch per delta-rule layer (prep
-        and scan together) when it applies, or always two."""
-        _check(_lib.kvm_set_fusion(self._h, FUSE_GDN, int(bool(enable))))
+        """kvm_set_plan(KVM_PLAN_GDN_FUSED): prep and chain of a delta-rule
+        layer in one launch when it applies, or always separate launches."""
+        _check(_lib.kvm_set_plan(self._h, PLAN_GDN_FUSED, int(bool(enable))))
+
+    def set_gdn_state_chain(self, enable=True):
+        """kvm_set_plan(KVM_PLAN_GDN_STATE_CHAIN): the chain carries only the
+        state and the outputs follow in a parallel pass (d_k = d_v = 128)."""
+        _check(_lib.kvm_set_plan(self._h, PLAN_GDN_STATE_CHAIN, int(bool(enable))))
 
     def debug_poke_canary(self):
         """kvm_debug_poke_canary (debug builds): spoil one canary byte."""

@@ -48,16 +48,18 @@ def test_tiny_round_via_separate_entry_points():
     _assert_errs(errs, what="tiny/entry points")
 
 
-def test_npc_shape_eight_chained_rounds():
+@pytest.mark.parametrize("state_chain", [True, False])
+def test_npc_shape_eight_chained_rounds(state_chain):
     """NPC-shaped stack (D 256, 16/2 heads, delta d 128, 3:1), shorter prefix so
     the oracle keeps up; 8 chained rounds, ragged tail (96 tokens: 1.5 chunks,
-    12 query tiles)."""
+    12 query tiles); both forms of the delta-rule chain."""
     from harness import Pair
     shape = W.npc_shape(4)
     N, M = 1024, 96
     w = W.Workload("npc-small", 11, shape, [N], 8)
     w.plan = [[(0.05, 1 + r % 4, M)] for r in range(8)]
     pair = Pair(shape, [N], w.capacity(), M, seed_index=w.index)
+    pair.ctx.set_gdn_state_chain(state_chain)
     for r in range(8):
         live = [pair.ctx.get_live(0)[0]]
         span_cu, sb, se, tails = W.round_plan(w, r, live)
@@ -263,18 +265,21 @@ def test_host_resident_round_equals_device_round(arena):
         assert live == [host.get_live(b)[0] for b in range(2)]
 
 
+@pytest.mark.parametrize("state_chain", [True, False])
 @pytest.mark.parametrize("n_chars,tails", [(1, [256]), (1, [1024]), (2, [130, 64]), (1, [1])])
-def test_delta_rule_launch_plans_agree(n_chars, tails):
+def test_delta_rule_launch_plans_agree(n_chars, tails, state_chain):
     """The delta-rule layer as one launch (prep workers publishing records
-    to scan blocks in the same grid) and as a prep launch followed by a scan
-    launch run the same arithmetic: outputs and states bit-identical, over
-    two rounds."""
+    to chain blocks in the same grid) and as separate launches run the same
+    arithmetic: outputs and states bit-identical, over two rounds, in both
+    forms of the chain."""
     import torch
     from paper_2609_18935_gb300 import kvm
     shape = W.ModelShape([W.GDN, W.GDN], 16, 2, 256, 64, 1e4, 16, 128, 128)
     mk = lambda: kvm.Context(shape.layer_kind, 16, 2, 256, 64, 1e4, 16, 128, 128, [2 * max(tails) + 64] * n_chars,
                              sum(tails))
     a, b = mk(), mk()
+    a.set_gdn_state_chain(state_chain)
+    b.set_gdn_state_chain(state_chain)
     b.set_gdn_fusion(False)
     w = W.Workload("plans", 55, shape, [0] * n_chars, 2)
     for ctx in (a, b):
