@@ -288,6 +288,16 @@ __device__ __forceinline__ uint32_t ld_shared_b32(uint32_t addr) {
     return v;
 }
 
+// One lane of a fully active warp (the lowest: the same lane at every call
+// while all 32 lanes take part).  Tensor-core instructions issued this way,
+// from a warp whose other lanes run the same loop, issue measurably faster
+// than from a lone lane in a divergent branch.
+__device__ __forceinline__ bool elect_one() {
+    uint32_t pred = 0;
+    asm volatile("{\n\t.reg .pred p;\n\telect.sync _|p, 0xffffffff;\n\tselp.b32 %0, 1, 0, p;\n\t}" : "=r"(pred));
+    return pred != 0;
+}
+
 // Barrier among `count` threads (a multiple of 32) of the block, id 1..15
 // (id 0 is __syncthreads).
 __device__ __forceinline__ void named_bar_sync(int id, int count) {

@@ -17,11 +17,14 @@
 //               of warp 11 the V tiles of each segment's keys, each through a
 //               three-stage ring (64 keys x D, 128-byte swizzle); separate
 //               warps keep the two rings from waiting on each other;
-//   warp 1      allocates TMEM; lane 0 issues S_j = Q K_j^T (tcgen05.mma,
+//   warp 1      allocates TMEM and issues S_j = Q K_j^T (tcgen05.mma,
 //               M 128, N 64, K D, Q read from TMEM) into two TMEM buffers;
-//   warp 10     lane 0 issues O += P_j V_j (M 128, N D, K 64) into the TMEM
+//   warp 10     issues O += P_j V_j (M 128, N D, K 64) into the TMEM
 //               accumulator.  Two issuers keep the S stream running ahead of
-//               the softmax while the PV stream follows it;
+//               the softmax while the PV stream follows it.  Each issuer warp
+//               runs its loop converged and one elected lane issues: a lone
+//               lane in a divergent branch issued the same MMAs at ~1.6x the
+//               cycles per instruction;
 //   warps 2-9   softmax: each query row is shared by the two warps that see
 //               its TMEM lane quarter (warp w reads lanes 32 (w mod 4) ..),
 //               one per 32-key half of S_j.  They stage the segment's Q tile
@@ -136,6 +139,12 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
     const int t_begin = p.cta_tile[cta], k_begin = p.cta_k[cta];
     const int t_end = p.cta_tile[cta + 1], k_end = p.cta_k[cta + 1];
     auto more = [&](int t, int k) { return t < t_end || (t == t_end && k < k_end); };
+    // A barrier wait of a whole issuer warp: lane 0 polls, the warp takes its result.
+    auto warp_wait = [&](uint32_t b, uint32_t parity, int tag) -> bool {
+        int r = 1;
+        if ((threadIdx.x & 31) == 0) r = mbar_wait(b, parity, abort_flag, p.err, kErrWait, p.diag, tag) ? 1 : 0;
+        return __shfl_sync(0xffffffffu, r, 0) != 0;
+    };
 
     if (tid == 0) {
         *abort_flag = 0;
@@ -212,25 +221,25 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
         __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------------------ S issuer
-        if (lane == 0) {
-            const uint32_t id_qk = idesc_bf16_f32(BM, BN, false);
-            const uint64_t k_desc0 = smem_desc_sw128(sK, 16, 1024);   // + (byte offset >> 4) per operand
-            bool ok = true;
-            int j = 0, seg = 0;
-            for (int t = t_begin, k = k_begin; ok && more(t, k); ++t, k = 0, ++seg) {
-                const Tile T = decode_tile(p, t);
-                const int n = ((t == t_end) ? k_end : T.nk) - k;
-                ok = mbar_wait(bar(Q_FULL), seg & 1, abort_flag, p.err, kErrWait, p.diag, 0x21 + 256 * seg);
-                for (int i = 0; i < n && ok; ++i, ++j) {
-                    const int sb = j & 1, st = j % STAGES;
-                    ok = mbar_wait(bar(K_FULL + st), (j / STAGES) & 1, abort_flag, p.err, kErrWait, p.diag, 0x22 + 256 * j);
-                    if (ok && j >= 2)
-                        ok = mbar_wait(bar(S_EMPTY + sb), ((j >> 1) - 1) & 1, abort_flag, p.err, kErrWait, p.diag,
-                                       0x23 + 256 * j);
-                    if (!ok) break;
-                    tc_fence_after();
-                    const uint64_t kd = k_desc0 + (uint64_t)((st * C::KV_BYTES) >> 4);
-                    const uint32_t d = tmem + C::TMEM_S + sb * BN;
+        // The whole warp runs the loop; lane 0 polls the barriers and an
+        // elected lane (lane 0 again) issues, so the descriptors stay warp-uniform.
+        const uint32_t id_qk = idesc_bf16_f32(BM, BN, false);
+        const uint64_t k_desc0 = smem_desc_sw128(sK, 16, 1024);   // + (byte offset >> 4) per operand
+        bool ok = true;
+        int j = 0, seg = 0;
+        for (int t = t_begin, k = k_begin; ok && more(t, k); ++t, k = 0, ++seg) {
+            const Tile T = decode_tile(p, t);
+            const int n = ((t == t_end) ? k_end : T.nk) - k;
+            ok = warp_wait(bar(Q_FULL), seg & 1, 0x21 + 256 * seg);
+            for (int i = 0; i < n && ok; ++i, ++j) {
+                const int sb = j & 1, st = j % STAGES;
+                ok = warp_wait(bar(K_FULL + st), (j / STAGES) & 1, 0x22 + 256 * j);
+                if (ok && j >= 2) ok = warp_wait(bar(S_EMPTY + sb), ((j >> 1) - 1) & 1, 0x23 + 256 * j);
+                if (!ok) break;
+                tc_fence_after();
+                const uint64_t kd = k_desc0 + (uint64_t)((st * C::KV_BYTES) >> 4);
+                const uint32_t d = tmem + C::TMEM_S + sb * BN;
+                if (elect_one()) {
 #pragma unroll
                     for (int ks = 0; ks < D / 16; ++ks)
                         mma_bf16_ts(d, tmem + C::TMEM_Q + ks * 8, kd + (uint64_t)((((ks >> 2) * (BN * 128)) + (ks & 3) * 32) >> 4),
@@ -238,36 +247,36 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
                     mma_commit(bar(S_FULL + sb));
                     mma_commit(bar(K_EMPTY + st));
                 }
+                __syncwarp();
             }
-            // every MMA issued by this thread completes before TMEM is released
-            mma_commit(bar(DRAIN_S));
-            volatile int never = 0;
-            mbar_wait(bar(DRAIN_S), 0, &never, p.err, kErrWait, nullptr, 0, 1000000000ull);
         }
+        // every MMA issued by this warp completes before TMEM is released
+        if (elect_one()) mma_commit(bar(DRAIN_S));
+        __syncwarp();
+        volatile int never = 0;
+        if (lane == 0) mbar_wait(bar(DRAIN_S), 0, &never, p.err, kErrWait, nullptr, 0, 1000000000ull);
         __syncwarp();
     } else if (warp == kPvWarp) {
-        // ------------------------------------------------------------ PV issuer
-        if (lane == 0) {
-            const uint32_t id_pv = idesc_bf16_f32(BM, D, true);
-            const uint64_t p_desc0 = smem_desc_sw128(sP, 16, 1024);
-            const uint64_t v_desc0 = smem_desc_sw128(sV, BN * 128, 1024);
-            bool ok = true;
-            int j = 0, seg = 0;
-            for (int t = t_begin, k = k_begin; ok && more(t, k); ++t, k = 0, ++seg) {
-                const Tile T = decode_tile(p, t);
-                const int n = ((t == t_end) ? k_end : T.nk) - k;
-                for (int i = 0; i < n && ok; ++i, ++j) {
-                    const int pb = j & 1, st = j % STAGES;
-                    ok = mbar_wait(bar(P_FULL + pb), (j >> 1) & 1, abort_flag, p.err, kErrWait, p.diag, 0x24 + 256 * j);
-                    if (ok)
-                        ok = mbar_wait(bar(V_FULL + st), (j / STAGES) & 1, abort_flag, p.err, kErrWait, p.diag, 0x25 + 256 * j);
-                    // the previous segment's O has been read out before it is overwritten
-                    if (ok && i == 0 && seg > 0)
-                        ok = mbar_wait(bar(O_EMPTY), (seg - 1) & 1, abort_flag, p.err, kErrWait, p.diag, 0x26 + 256 * seg);
-                    if (!ok) break;
-                    tc_fence_after();
-                    const uint64_t pd = p_desc0 + (uint64_t)((pb * C::P_BYTES) >> 4);
-                    const uint64_t vd = v_desc0 + (uint64_t)((st * C::KV_BYTES) >> 4);
+        // ------------------------------------------------------------ PV issuer (same warp discipline)
+        const uint32_t id_pv = idesc_bf16_f32(BM, D, true);
+        const uint64_t p_desc0 = smem_desc_sw128(sP, 16, 1024);
+        const uint64_t v_desc0 = smem_desc_sw128(sV, BN * 128, 1024);
+        bool ok = true;
+        int j = 0, seg = 0;
+        for (int t = t_begin, k = k_begin; ok && more(t, k); ++t, k = 0, ++seg) {
+            const Tile T = decode_tile(p, t);
+            const int n = ((t == t_end) ? k_end : T.nk) - k;
+            for (int i = 0; i < n && ok; ++i, ++j) {
+                const int pb = j & 1, st = j % STAGES;
+                ok = warp_wait(bar(P_FULL + pb), (j >> 1) & 1, 0x24 + 256 * j);
+                if (ok) ok = warp_wait(bar(V_FULL + st), (j / STAGES) & 1, 0x25 + 256 * j);
+                // the previous segment's O has been read out before it is overwritten
+                if (ok && i == 0 && seg > 0) ok = warp_wait(bar(O_EMPTY), (seg - 1) & 1, 0x26 + 256 * seg);
+                if (!ok) break;
+                tc_fence_after();
+                const uint64_t pd = p_desc0 + (uint64_t)((pb * C::P_BYTES) >> 4);
+                const uint64_t vd = v_desc0 + (uint64_t)((st * C::KV_BYTES) >> 4);
+                if (elect_one()) {
 #pragma unroll
                     for (int ks = 0; ks < BN / 16; ++ks)
                         mma_bf16(tmem + C::TMEM_O, pd + (uint64_t)((ks * 32) >> 4), vd + (uint64_t)((ks * 16 * 128) >> 4), id_pv,
@@ -275,12 +284,17 @@ __global__ void __launch_bounds__(kThreads, 1) tail_attention_tc_kernel(const __
                     mma_commit(bar(PV_DONE + pb));
                     mma_commit(bar(V_EMPTY + st));
                 }
-                if (ok) mma_commit(bar(O_FINAL));
+                __syncwarp();
             }
-            mma_commit(bar(DRAIN_PV));
-            volatile int never = 0;
-            mbar_wait(bar(DRAIN_PV), 0, &never, p.err, kErrWait, nullptr, 0, 1000000000ull);
+            if (ok) {
+                if (elect_one()) mma_commit(bar(O_FINAL));
+                __syncwarp();
+            }
         }
+        if (elect_one()) mma_commit(bar(DRAIN_PV));
+        __syncwarp();
+        volatile int never = 0;
+        if (lane == 0) mbar_wait(bar(DRAIN_PV), 0, &never, p.err, kErrWait, nullptr, 0, 1000000000ull);
         __syncwarp();
     } else {
         // ------------------------------------------------------------ softmax + epilogue
