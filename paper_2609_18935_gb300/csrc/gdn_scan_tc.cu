@@ -1500,9 +1500,253 @@ __device__ __forceinline__ void gdn_scan_run(const GdnParams& p, const FuseCtl& 
     }
 }
 
+// Scan of a slice of at most 32 d_v rows with hi | lo packed side by side in
+// one 64-column operand.  The MMAs of the chain are short (N <= 64), so their
+// cost is per instruction rather than per column: [W; Q'] (hi, then lo)
+// against [S_hi | S_lo] takes 2 DK/16 MMAs instead of 3 DK/16, and
+// K^T [wE_hi | wE_lo] takes C/16 instead of 2 C/16.  Each product's two
+// halves land in columns c and 32 + c of its accumulator and are added when
+// read.  The state stays fp32 in the threads' registers (thread (row,
+// column half) holds S^T[row][16 columns]); TMEM holds only the two
+// products:
+//     D1 = [W; Q'] [S_hi | S_lo]             E = w (U - D1a - D1b),  O = A U + D1a + D1b
+//     D2 = K^T [wE_hi | wE_lo]               S^T = G_C S^T + D2a + D2b
+template <int DK>
+__device__ __forceinline__ void gdn_scan_packed_run(const GdnParams& p, const FuseCtl& fc, int b, int h, int r0) {
+    using G = ScanCfg<DK>;
+    using R = Rec<DK>;
+    constexpr int CW = 16;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    const uint32_t sb = smem_u32(smem);
+    auto V4 = [&](uint32_t off) -> uint4& { return *reinterpret_cast<uint4*>(smem + off); };
+    constexpr uint32_t oS = G::OFF_S;                // [S_hi | S_lo]: DK rows of 128 bytes; [wE_hi | wE_lo] (C rows) aliases it
+    constexpr uint32_t T_D1 = 0, T_D2 = 128;         // 64 columns each
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + G::OFF_BAR);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + G::OFF_BAR + 32);
+    const uint32_t mbar = smem_u32(&bars[0]);
+    const uint32_t bar_wq = smem_u32(&bars[1]), bar_k = smem_u32(&bars[2]), bar_u = smem_u32(&bars[3]);
+    const float* Us = reinterpret_cast<const float*>(smem + G::OFF_U);
+    __shared__ volatile int abort_flag;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int q4 = warp & 3, hf = warp >> 2;
+    const int row = q4 * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    const int dvs = p.dv_slice;                      // <= 32
+    const GdnChar ch = p.ch[b];
+    if (ch.M <= 0) return;                           // uniform per block; touches no memory
+    const int H = p.H, dv = p.dv;
+    const int nch = (ch.M + C - 1) / C;
+    const uint32_t ubytes = 128u * dvs * 4u;
+    const int64_t uslice = R::uau_off() + (int64_t)r0 * 128 * 4;
+    float* Sg = p.S + ((int64_t)b * H + h) * dv * DK;
+    const int rc = hf * CW;                          // columns rc .. rc + 15 of the slice
+    const bool cols = hf < 2 && rc < dvs;            // uniform per warp (fused blocks: warps 8.. have none)
+    auto rec_of = [&](int i) -> const uint8_t* { return p.work + ((int64_t)(ch.chunk_off + i) * H + h) * p.rec_bytes; };
+
+    if (tid == 0) {
+        abort_flag = 0;
+        mbar_init(mbar, 1);
+        mbar_init(bar_wq, 1);
+        mbar_init(bar_k, 1);
+        mbar_init(bar_u, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(tmem_slot), 256);
+        tmem_relinquish();
+    }
+    // columns no thread owns (slices narrower than 32) stay zero
+    for (int i = tid; i < DK * 128 / 16; i += blockDim.x) V4(oS + 16 * i) = make_uint4(0, 0, 0, 0);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    // row `row` of S^T, hi at column c and lo at column 32 + c of the operand
+    auto write_s = [&](int r, const float* x) {
+#pragma unroll
+        for (int j8 = 0; j8 < CW; j8 += 8) {
+            if (rc + j8 < dvs) {
+                uint4 hi, lo;
+                split8(x + j8, hi, lo);
+                V4(oS + sw128_off16(r, rc + j8, DK)) = hi;
+                V4(oS + sw128_off16(r, 32 + rc + j8, DK)) = lo;
+            }
+        }
+    };
+    float sreg[CW];
+#pragma unroll
+    for (int j = 0; j < CW; ++j)                     // all loads before any use
+        sreg[j] = (cols && row < DK && rc + j < dvs) ? Sg[(int64_t)(r0 + rc + j) * DK + row] : 0.f;
+    if (cols && row < DK) write_s(row, sreg);
+    // The state slice comes from an earlier round (or kvm_set_state), which
+    // completed before the prep kernel this launch follows had started, so
+    // it is staged before waiting for that kernel; its records are not.
+    if (!fc.flags) {                                 // the fused kernel waited already
+        grid_dependency_wait();
+        grid_dependents_launch();
+    }
+    if (tid == 0 && wait_record(fc, (int64_t)ch.chunk_off * H + h, &abort_flag, p.err, p.diag, 0x5f)) {
+        mbar_arrive_expect_tx(bar_wq, G::WQ);
+        bulk_load(sb + G::OFF_WQ, rec_of(0), G::WQ, bar_wq);
+        mbar_arrive_expect_tx(bar_k, G::KI);
+        bulk_load(sb + G::OFF_K, rec_of(0) + G::WQ, G::KI, bar_k);
+        mbar_arrive_expect_tx(bar_u, ubytes);
+        bulk_load(sb + G::OFF_U, rec_of(0) + uslice, ubytes, bar_u);
+    }
+
+    uint32_t phase = 0;
+    bool ok = true;
+    auto mma_wait = [&]() -> bool {
+        bool r = true;
+        if (tid == 0) r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait, p.diag, 0x50);
+        phase ^= 1;
+        r = __syncthreads_and(r);
+        tc_fence_after();
+        return r;
+    };
+    auto issue_begin = [&]() { fence_proxy_async_smem(); tc_fence_before(); __syncthreads(); };
+    const uint32_t id_1 = idesc_bf16_f32(128, 64, true);           // B = [S_hi | S_lo], MN-major
+    const uint32_t id_2 = idesc_bf16_f32(128, 64, true, true);     // A = K, B = [wE_hi | wE_lo], both MN-major
+    const uint32_t kq_region = 128 * 128;
+    issue_begin();
+
+    for (int i = 0; i < nch && ok; ++i) {
+        const int n = min(C, ch.M - i * C);
+        const int64_t tok0 = ch.tail_off + (int64_t)i * C;
+        const uint8_t* rec = rec_of(i);
+        const float* misc = reinterpret_cast<const float*>(rec + R::misc_off(dv));
+        const float wt = __ldcg(misc + (row & 63));
+        const float gC = __ldcg(misc + C);
+        // ---------------------------------------------------------------- D1 = [W; Q'] [S_hi | S_lo]
+        if (tid == 0 && mbar_wait(bar_wq, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x51 + 256 * i)) {
+            tc_fence_after();
+#pragma unroll
+            for (int ks = 0; ks < DK / 16; ++ks) {
+                const uint32_t ao = (ks >> 2) * kq_region + (ks & 3) * 32;
+                const uint64_t bs = smem_desc_sw128(sb + oS + ks * 2048, DK * 128, 1024);
+                mma_bf16(tmem + T_D1, smem_desc_sw128(sb + G::OFF_WQ + ao, 16, 1024), bs, id_1, ks > 0);
+                mma_bf16(tmem + T_D1, smem_desc_sw128(sb + G::OFF_WQ + (uint32_t)R::WQH + ao, 16, 1024), bs, id_1, 1u);
+            }
+            mma_commit(mbar);
+        }
+        ok = mma_wait();
+        if (!ok) break;
+        if (tid == 0 && i + 1 < nch &&
+            wait_record(fc, (int64_t)(ch.chunk_off + i + 1) * H + h, &abort_flag, p.err, p.diag, 0x5e + 256 * i)) {
+            mbar_arrive_expect_tx(bar_wq, G::WQ);
+            bulk_load(sb + G::OFF_WQ, rec_of(i + 1), G::WQ, bar_wq);
+        }
+        // ---------------------------------------------------------------- E (rows < 64) and O (rows >= 64)
+        const bool u_ok = mbar_wait(bar_u, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x52 + 256 * i);
+        if (cols) {
+            const int t = row & 63;
+            uint32_t da[CW], db[CW];
+            tmem_ldw<CW>(tmem + lane_off + T_D1 + rc, da);
+            tmem_ldw<CW>(tmem + lane_off + T_D1 + 32 + rc, db);
+            float u[CW];
+#pragma unroll
+            for (int j4 = 0; j4 < CW; j4 += 4) {
+                const float4 f = *reinterpret_cast<const float4*>(Us + uau_idx(row, rc + j4));
+                u[j4] = f.x; u[j4 + 1] = f.y; u[j4 + 2] = f.z; u[j4 + 3] = f.w;
+            }
+            tmem_ld_wait();
+            float d[CW];
+#pragma unroll
+            for (int j = 0; j < CW; ++j) d[j] = __uint_as_float(da[j]) + __uint_as_float(db[j]);
+            if (row < 64) {
+                float e[CW];
+#pragma unroll
+                for (int j = 0; j < CW; ++j) e[j] = wt * (u[j] - d[j]);
+#pragma unroll
+                for (int j8 = 0; j8 < CW; j8 += 8) {
+                    if (rc + j8 < dvs) {
+                        uint4 hi, lo;
+                        split8(e + j8, hi, lo);
+                        V4(oS + sw128_off16(t, rc + j8, C)) = hi;          // [wE_hi | wE_lo] aliases the S operand
+                        V4(oS + sw128_off16(t, 32 + rc + j8, C)) = lo;
+                    }
+                }
+            } else if (t < n) {
+                __nv_bfloat16* o = p.out + ((tok0 + t) * H + h) * dv + r0 + rc;
+#pragma unroll
+                for (int j8 = 0; j8 < CW; j8 += 8) {
+                    if (rc + j8 < dvs) {
+                        uint4 w4;
+                        uint32_t* ww = reinterpret_cast<uint32_t*>(&w4);
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            ww[e] = pack_bf16x2(u[j8 + 2 * e] + d[j8 + 2 * e], u[j8 + 2 * e + 1] + d[j8 + 2 * e + 1]);
+                        *reinterpret_cast<uint4*>(o + j8) = w4;
+                    }
+                }
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        ok = __syncthreads_and(u_ok);
+        if (!ok) break;
+        if (tid == 0 && i + 1 < nch && !abort_flag) {
+            mbar_arrive_expect_tx(bar_u, ubytes);
+            bulk_load(sb + G::OFF_U, rec_of(i + 1) + uslice, ubytes, bar_u);
+        }
+        // ---------------------------------------------------------------- D2 = K^T [wE_hi | wE_lo]
+        if (tid == 0 && mbar_wait(bar_k, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x53 + 256 * i)) {
+            tc_fence_after();
+#pragma unroll
+            for (int ks = 0; ks < C / 16; ++ks)
+                mma_bf16(tmem + T_D2, smem_desc_sw128(sb + G::OFF_K + ks * 2048, C * 128, 1024),
+                         smem_desc_sw128(sb + oS + ks * 2048, C * 128, 1024), id_2, ks > 0);
+            mma_commit(mbar);
+        }
+        ok = mma_wait();
+        if (!ok) break;
+        if (tid == 0 && i + 1 < nch && !abort_flag) {
+            mbar_arrive_expect_tx(bar_k, G::KI);
+            bulk_load(sb + G::OFF_K, rec_of(i + 1) + G::WQ, G::KI, bar_k);
+        }
+        // ---------------------------------------------------------------- S^T = G_C S^T + D2a + D2b
+        if (cols) {
+            uint32_t da[CW], db[CW];
+            tmem_ldw<CW>(tmem + lane_off + T_D2 + rc, da);
+            tmem_ldw<CW>(tmem + lane_off + T_D2 + 32 + rc, db);
+            tmem_ld_wait();
+            if (row < DK) {
+#pragma unroll
+                for (int j = 0; j < CW; ++j) sreg[j] = fmaf(gC, sreg[j], __uint_as_float(da[j]) + __uint_as_float(db[j]));
+                write_s(row, sreg);
+            }
+        }
+        issue_begin();
+    }
+    if (ok) {
+        if (cols && row < DK) {
+#pragma unroll
+            for (int j = 0; j < CW; ++j)
+                if (rc + j < dvs) Sg[(int64_t)(r0 + rc + j) * DK + row] = sreg[j];
+        }
+    } else if (tid == 0) {
+        // let outstanding record copies land before the block exits
+        volatile int never = 0;
+        const uint32_t bs3[3] = {bar_wq, bar_k, bar_u};
+        for (int k = 0; k < 3; ++k) {
+            mbar_wait(bs3[k], 0, &never, p.err, kErrWait, nullptr, 0, 20000000ull);
+            mbar_wait(bs3[k], 1, &never, p.err, kErrWait, nullptr, 0, 20000000ull);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 256);
+    }
+}
+
 template <int DK, int CW>
 __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_constant__ GdnParams p) {
-    gdn_scan_run<DK, CW>(p, FuseCtl{nullptr, 0}, blockIdx.z, blockIdx.y, blockIdx.x * p.dv_slice);
+    if constexpr (CW == 16) gdn_scan_packed_run<DK>(p, FuseCtl{nullptr, 0}, blockIdx.z, blockIdx.y, blockIdx.x * p.dv_slice);
+    else gdn_scan_run<DK, CW>(p, FuseCtl{nullptr, 0}, blockIdx.z, blockIdx.y, blockIdx.x * p.dv_slice);
 }
 
 // ============================================================================
@@ -1523,7 +1767,7 @@ __global__ void __launch_bounds__(kPrepThreads, 1) gdn_fused_kernel(const __grid
     const int x = blockIdx.x;
     if (x < p.n_scan) {
         const int slices = p.dv / p.dv_slice;
-        gdn_scan_run<DK, CW>(p, fc, x / (slices * p.H), (x / slices) % p.H, (x % slices) * p.dv_slice);
+        gdn_scan_packed_run<DK>(p, fc, x / (slices * p.H), (x / slices) % p.H, (x % slices) * p.dv_slice);
     } else {
         gdn_prep_run<DK>(p, fc, x - p.n_scan, gridDim.x - p.n_scan);
     }
