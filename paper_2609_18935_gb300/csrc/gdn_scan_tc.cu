@@ -1536,6 +1536,11 @@ __device__ __forceinline__ void gdn_scan_packed_run(const GdnParams& p, const Fu
     const int dvs = p.dv_slice;                      // <= 32
     const GdnChar ch = p.ch[b];
     if (ch.M <= 0) return;                           // uniform per block; touches no memory
+    // The scan runs on warps 0-7 and synchronises them with barrier 1 of 256
+    // threads; the other warps of a fused launch's 512-thread block leave.
+    if (warp >= kThreads / 32) return;
+    auto sync = [&]() { named_bar_sync(1, kThreads); };
+    auto sync_and = [&](bool x) { return named_bar_and(1, kThreads, x); };
     const int H = p.H, dv = p.dv;
     const int nch = (ch.M + C - 1) / C;
     const uint32_t ubytes = 128u * dvs * 4u;
@@ -1558,9 +1563,9 @@ __device__ __forceinline__ void gdn_scan_packed_run(const GdnParams& p, const Fu
         tmem_relinquish();
     }
     // columns no thread owns (slices narrower than 32) stay zero
-    for (int i = tid; i < DK * 128 / 16; i += blockDim.x) V4(oS + 16 * i) = make_uint4(0, 0, 0, 0);
+    for (int i = tid; i < DK * 128 / 16; i += kThreads) V4(oS + 16 * i) = make_uint4(0, 0, 0, 0);
     tc_fence_before();
-    __syncthreads();
+    sync();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     // row `row` of S^T, hi at column c and lo at column 32 + c of the operand
@@ -1602,11 +1607,11 @@ __device__ __forceinline__ void gdn_scan_packed_run(const GdnParams& p, const Fu
         bool r = true;
         if (tid == 0) r = mbar_wait(mbar, phase, &abort_flag, p.err, kErrWait, p.diag, 0x50);
         phase ^= 1;
-        r = __syncthreads_and(r);
+        r = sync_and(r);
         tc_fence_after();
         return r;
     };
-    auto issue_begin = [&]() { fence_proxy_async_smem(); tc_fence_before(); __syncthreads(); };
+    auto issue_begin = [&]() { fence_proxy_async_smem(); tc_fence_before(); sync(); };
     const uint32_t id_1 = idesc_bf16_f32(128, 64, true);           // B = [S_hi | S_lo], MN-major
     const uint32_t id_2 = idesc_bf16_f32(128, 64, true, true);     // A = K, B = [wE_hi | wE_lo], both MN-major
     const uint32_t kq_region = 128 * 128;
@@ -1639,7 +1644,7 @@ __device__ __forceinline__ void gdn_scan_packed_run(const GdnParams& p, const Fu
             bulk_load(sb + G::OFF_WQ, rec_of(i + 1), G::WQ, bar_wq);
         }
         // ---------------------------------------------------------------- E (rows < 64) and O (rows >= 64)
-        const bool u_ok = mbar_wait(bar_u, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x52 + 256 * i);
+        const bool u_ok = !cols || mbar_wait(bar_u, i & 1, &abort_flag, p.err, kErrWait, p.diag, 0x52 + 256 * i);
         if (cols) {
             const int t = row & 63;
             uint32_t da[CW], db[CW];
@@ -1685,7 +1690,7 @@ __device__ __forceinline__ void gdn_scan_packed_run(const GdnParams& p, const Fu
         }
         fence_proxy_async_smem();
         tc_fence_before();
-        ok = __syncthreads_and(u_ok);
+        ok = sync_and(u_ok);
         if (!ok) break;
         if (tid == 0 && i + 1 < nch && !abort_flag) {
             mbar_arrive_expect_tx(bar_u, ubytes);
@@ -1736,7 +1741,7 @@ __device__ __forceinline__ void gdn_scan_packed_run(const GdnParams& p, const Fu
         }
     }
     tc_fence_before();
-    __syncthreads();
+    sync();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc(tmem, 256);
