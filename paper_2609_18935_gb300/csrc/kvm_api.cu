@@ -139,6 +139,9 @@ struct kvm_ctx {
     // that come before the first attention layer (it touches only the KV cache)
     cudaStream_t compact_stream = nullptr;
     cudaEvent_t ev_round = nullptr, ev_compacted = nullptr;
+    // per attention layer: the main stream reached the layers its compaction
+    // runs beside, and that compaction is done
+    std::vector<cudaEvent_t> ev_piece_go, ev_piece_done;
     std::vector<cudaEvent_t> ev_in, ev_done;   // per layer: inputs landed, outputs written
     double inv_freq[kMaxRotaryHalf] = {};
     CUtensorMap tmap_k, tmap_v;           // TMA maps of K, V (attention layers only)
@@ -203,6 +206,8 @@ void free_all(kvm_ctx* c) {
     if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
     if (c->ev_round) cudaEventDestroy(c->ev_round);
     if (c->ev_compacted) cudaEventDestroy(c->ev_compacted);
+    for (cudaEvent_t e : c->ev_piece_go) if (e) cudaEventDestroy(e);
+    for (cudaEvent_t e : c->ev_piece_done) if (e) cudaEventDestroy(e);
     if (c->compact_stream) cudaStreamDestroy(c->compact_stream);
     for (cudaEvent_t e : c->ev) cudaEventDestroy(e);
     c->ev.clear();
@@ -544,6 +549,12 @@ extern "C" kvm_status kvm_create(const kvm_model_desc* m, int32_t n_chars, const
         if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&c->compact_stream, cudaStreamNonBlocking);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_round, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_compacted, cudaEventDisableTiming);
+        c->ev_piece_go.assign(c->n_attn, nullptr);
+        c->ev_piece_done.assign(c->n_attn, nullptr);
+        for (int a = 0; a < c->n_attn && e == cudaSuccess; ++a) {
+            e = cudaEventCreateWithFlags(&c->ev_piece_go[a], cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_piece_done[a], cudaEventDisableTiming);
+        }
         c->ev_in.assign(c->n_layers, nullptr);
         c->ev_done.assign(c->n_layers, nullptr);
         for (int l = 0; l < c->n_layers && e == cudaSuccess; ++l) {
@@ -1501,51 +1512,79 @@ kvm_status update_round_impl(kvm_ctx* c, const kvm_round* r, void* stream) {
         }
     }
     // Compaction changes only the attention layers' caches.  When recurrent
-    // layers come before the first attention layer, it runs on the compaction
-    // stream beside them (after everything already queued on s), and s joins
-    // it at the first attention layer (measured: 6.68 against 6.71 ms for the
-    // long round when joining one layer earlier).  (One launch for all
-    // attention layers, one-shot blocks: launches per layer have too few
-    // blocks each, and a persistent grid keeps the recurrent layers' launches
-    // off the SMs it holds; both slowed the layers they run beside.)
+    // layers come before the first attention layer, each attention layer's
+    // cache is compacted on the compaction stream beside the recurrent layers
+    // that precede it (after the attention layer before them has finished),
+    // and s joins that piece at the attention layer; the positions go with
+    // the first piece.  Otherwise one launch on s compacts every layer.
     int first_attn = c->n_layers;
     for (int l = c->n_layers - 1; l >= 0; --l)
         if (c->kind[l] == KVM_LAYER_ATTN) first_attn = l;
     const bool side = first_attn > 0 && first_attn < c->n_layers;
-    {
-        SpanPlan pl;
-        st = plan_spans(c, r->span_cu, r->span_begin, r->span_end, pl);
-        if (st) return st;
-        cudaStream_t cs = side ? c->compact_stream : s;
-        if (side) {
-            CUDA_TRY(cudaEventRecord(c->ev_round, s));
-            CUDA_TRY(cudaStreamWaitEvent(cs, c->ev_round, 0));
+    SpanPlan pl;
+    st = plan_spans(c, r->span_cu, r->span_begin, r->span_end, pl);
+    if (st) return st;
+    // piece a runs beside the layers from piece_at[a] up to its attention layer
+    std::vector<int> piece_at(c->n_attn, 0);
+    for (int l = 0, prev = -1; l < c->n_layers; ++l)
+        if (c->kind[l] == KVM_LAYER_ATTN) {
+            piece_at[c->attn_idx[l]] = prev + 1;
+            prev = l;
         }
+    std::vector<char> piece_out(c->n_attn, 0);       // launched and not yet joined
+    auto launch_piece = [&](int a) -> kvm_status {
         NvtxRange range("kv_compact");
-        // the gather map depends on the plan only; it goes first so that the
-        // events of the compactions cover it
-        st = launch_gather(c, pl, r->gather_out, cs);
+        CUDA_TRY(cudaEventRecord(c->ev_piece_go[a], s));
+        CUDA_TRY(cudaStreamWaitEvent(c->compact_stream, c->ev_piece_go[a], 0));
+        if (a == 0) {
+            // the gather map depends on the plan only; the first piece's event covers it
+            const kvm_status g = launch_gather(c, pl, r->gather_out, c->compact_stream);
+            if (g) return g;
+        }
+        const kvm_status e = launch_compaction(c, pl, c->compact_stream, a, a + 1, a == 0);
+        if (e) return e;
+        CUDA_TRY(cudaEventRecord(c->ev_piece_done[a], c->compact_stream));
+        piece_out[a] = 1;
+        return KVM_OK;
+    };
+    auto join_piece = [&](int a) -> cudaError_t {
+        if (!piece_out[a]) return cudaSuccess;
+        piece_out[a] = 0;
+        return cudaStreamWaitEvent(s, c->ev_piece_done[a], 0);
+    };
+    auto join = [&]() -> cudaError_t {                // every piece launched so far
+        for (int a = 0; a < c->n_attn; ++a) {
+            const cudaError_t e = join_piece(a);
+            if (e != cudaSuccess) return e;
+        }
+        return cudaSuccess;
+    };
+    if (!side) {
+        NvtxRange range("kv_compact");
+        st = launch_gather(c, pl, r->gather_out, s);
         if (st) return st;
-        st = launch_compaction(c, pl, cs, 0, c->n_attn, true);
+        st = launch_compaction(c, pl, s, 0, c->n_attn, true);
         if (st) return st;
-        if (side) CUDA_TRY(cudaEventRecord(c->ev_compacted, cs));
-        apply_plan(c, pl, r->span_cu, r->span_begin, r->span_end);
     }
+    apply_plan(c, pl, r->span_cu, r->span_begin, r->span_end);
     const bool with_pos = r->tail_pos && total > 0 && c->n_attn > 0;
     if (with_pos) {
         st = stage_positions(c, r->tail_pos, total, c->tail_pos_dev, s);
         if (st) return st;
     }
-    const int join_at = first_attn;
-    bool joined = !side;
-    auto join = [&]() -> cudaError_t {
-        if (joined) return cudaSuccess;
-        joined = true;
-        return cudaStreamWaitEvent(s, c->ev_compacted, 0);
-    };
     for (int l = 0; l < c->n_layers; ++l) {
         const bool attn = c->kind[l] == KVM_LAYER_ATTN;
-        if (l == join_at) CUDA_TRY(join());
+        if (side) {
+            for (int a = 0; a < c->n_attn; ++a)
+                if (piece_at[a] == l) {
+                    st = launch_piece(a);
+                    if (st) {
+                        join();
+                        return st;
+                    }
+                }
+            if (attn) CUDA_TRY(join_piece(c->attn_idx[l]));
+        }
         const void *q = r->q[l], *k = r->k[l], *v = r->v[l];
         const float *al = attn ? nullptr : r->alpha[l], *be = attn ? nullptr : r->beta[l];
         void* out = r->out[l];
