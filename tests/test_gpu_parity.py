@@ -298,3 +298,26 @@ def test_delta_rule_launch_plans_agree(n_chars, tails, state_chain):
         for l in (0, 1):
             assert torch.equal(outs[0][l].view(torch.int16), outs[1][l].view(torch.int16)), (r, l)
             assert torch.equal(a.get_state(l), b.get_state(l)), (r, l)
+
+
+@pytest.mark.parametrize("pattern", ["GAAGGA", "AGA"])
+def test_compaction_scheduling_over_layer_patterns(pattern):
+    """Layer orders that exercise how a round places its compactions: with
+    recurrent layers before the first attention layer, each attention layer's
+    cache is compacted in a launch of its own beside the layers before it
+    (here two attention layers are also adjacent, so one such launch runs
+    right at its layer); with an attention layer first, one launch on the
+    caller's stream compacts every layer.  Two chained rounds against the
+    oracle, caches bit-exact, outputs and states within the bar."""
+    from harness import Pair
+    kinds = [W.GDN if ch == "G" else W.ATTN for ch in pattern]
+    shape = W.ModelShape(kinds, 8, 2, 64, 64, 1.0e4, 8, 64, 64)
+    N = [300, 520]
+    w = W.Workload("sched-" + pattern, 61, shape, N, 2)
+    w.plan = [[(0.08, 3, 70), (0.05, 2, 40)], [(0.06, 2, 33), (0.04, 1, 90)]]
+    pair = Pair(shape, N, w.capacity(), 70 + 90, seed_index=w.index)
+    for rnd in range(2):
+        live = [pair.ctx.get_live(b)[0] for b in range(2)]
+        span_cu, sb, se, tails = W.round_plan(w, rnd, live)
+        errs = pair.run_round(span_cu, sb, se, tails, W.tail_inputs(w, rnd, tails))
+        _assert_errs(errs, what=f"{pattern} round {rnd}")
