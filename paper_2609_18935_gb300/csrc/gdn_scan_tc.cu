@@ -282,10 +282,8 @@ __device__ __forceinline__ void gdn_prep_run(const GdnParams& p, const FuseCtl& 
         tmem_alloc(smem_u32(tmem_slot), 512);
         tmem_relinquish();
     }
-    if (!fc.flags) {                                 // the fused kernel waited already
-        grid_dependency_wait();
-        grid_dependents_launch();
-    }
+    grid_dependency_wait();                          // the chunk inputs may come from the previous grid
+    grid_dependents_launch();
     uint32_t phase = 0;
     for (int u = u0; u < n_units; u += ustride) {
     // with two parts per (chunk, head) both solve for X; part 0 writes the
@@ -1588,10 +1586,8 @@ __device__ __forceinline__ void gdn_scan_packed_run(const GdnParams& p, const Fu
     // The state slice comes from an earlier round (or kvm_set_state), which
     // completed before the prep kernel this launch follows had started, so
     // it is staged before waiting for that kernel; its records are not.
-    if (!fc.flags) {                                 // the fused kernel waited already
-        grid_dependency_wait();
-        grid_dependents_launch();
-    }
+    grid_dependency_wait();
+    grid_dependents_launch();
     if (tid == 0 && wait_record(fc, (int64_t)ch.chunk_off * H + h, &abort_flag, p.err, p.diag, 0x5f)) {
         mbar_arrive_expect_tx(bar_wq, G::WQ);
         bulk_load(sb + G::OFF_WQ, rec_of(0), G::WQ, bar_wq);
@@ -1769,8 +1765,7 @@ __global__ void __launch_bounds__(kThreads, 1) gdn_scan_kernel(const __grid_cons
 // ============================================================================
 template <int DK, int CW>
 __global__ void __launch_bounds__(kPrepThreads, 1) gdn_fused_kernel(const __grid_constant__ GdnParams p) {
-    grid_dependency_wait();
-    grid_dependents_launch();
+    // each role waits for the previous grid after its own set-up (below)
     const FuseCtl fc{p.flags, p.epoch};
     const int x = blockIdx.x;
     if (x < p.n_scan) {
