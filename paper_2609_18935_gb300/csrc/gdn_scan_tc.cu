@@ -365,7 +365,6 @@ __device__ __forceinline__ void gdn_prep_run(const GdnParams& p, const FuseCtl& 
             float* misc = reinterpret_cast<float*>(rec + R::misc_off(dv));
             misc[tid] = tid < n ? bs[tid] * expf(gs[n - 1] - gs[tid]) : 0.f;     // w_j
             if (tid == 0) misc[C] = expf(gs[n - 1]);                            // G_C
-            if (fc.flags) __threadfence();                                      // before the record's flag
         }
     }
     bool ok = true;
@@ -668,6 +667,9 @@ __device__ __forceinline__ void gdn_prep_run(const GdnParams& p, const FuseCtl& 
             bulk_wait_read();
         }
     }
+    // fused: w and G_C (plain stores above) are ordered before the record's
+    // flag; fencing here, long after the stores, costs little
+    if (fc.flags && do_u && tid < C) __threadfence();
     tc_fence_before();
     __syncthreads();                                 // the staging area is free for the next unit
     tc_fence_after();
