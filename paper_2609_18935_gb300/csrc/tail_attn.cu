@@ -166,6 +166,87 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
     if (threadIdx.x == 0) p.pos[slot] = (int32_t)pos;
 }
 
+// grid (n_split_tiles, kRows * D / 4 / 256): the x-th query tile that several
+// attention blocks share.  Block cb = split_cb[x] is the first to start
+// inside the tile, so its partials are in the slots of blocks c0 = cb - 1 ..
+// c1 (the last block that starts inside the tile): c0's last segment (slot
+// 2 c0 + 1, or 2 c0 when the tile is also c0's first segment) and the first
+// segments 2 c of the others.  A thread owns four columns of one row (rows
+// fastest across threads, as in the partial layout) and merges the partials
+// online, two at a time, each batch's (max, sum) pairs and O pieces loaded
+// together.
+// At most 36 registers a thread keep seven blocks on an SM, so that the
+// grid of a round with up to 33 shared tiles (x 32 blocks at head_dim 256)
+// runs in one wave.
+__global__ void __launch_bounds__(256, 7) attn_combine_piece_kernel(const __grid_constant__ AttnParams p) {
+    grid_dependency_wait();
+    grid_dependents_launch();
+    const int cb = p.split_cb[blockIdx.x];
+    const int t = p.cta_tile[cb];
+    const int c0 = cb - 1;
+    int c1 = cb;
+    while (c1 + 1 < p.n_ctas && p.cta_tile[c1 + 1] == t && p.cta_k[c1 + 1] > 0) ++c1;
+    const int slot0 = (p.cta_tile[c0] == t) ? 2 * c0 : 2 * c0 + 1;
+    const int n_parts = c1 - c0 + 1;
+
+    int lo = 0, hi = p.n_chars - 1;                                // last b with tile_off <= t
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (p.ch[mid].tile_off <= t) lo = mid; else hi = mid - 1;
+    }
+    const AttnChar& c = p.ch[lo];
+    const int local = t - c.tile_off;
+    const int kvh = local / c.n_qtiles, qt = local % c.n_qtiles;
+    const int D = p.D;
+    const int item = blockIdx.y * blockDim.x + threadIdx.x;        // (4-column piece, row): rows fastest
+    const int r = item % kRows;
+    const int piece = item / kRows;
+    if (piece >= D / 4) return;
+    const int cg = piece >> 3, q4 = piece & 7;
+    const int tok = qt * p.tok_per_tile + r / p.g;
+    if (tok >= c.M) return;
+    __nv_bfloat16* o = p.out + ((int64_t)(c.tail_off + tok) * p.Hq + kvh * p.g + (r % p.g)) * D + cg * 32 + q4 * 4;
+    // this thread's piece of slot s: po + s * D * kRows floats; its (max, sum): pm + s * 2 kRows
+    const float* po = p.part_o + ((cg * 8 + q4) * kRows + r) * 4;
+    const float* pm = p.part_ml + r * 2;
+    const int sstride = D * kRows;
+    constexpr int kBatch = 2;
+    float mx = -INFINITY, den = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int q0 = 0; q0 < n_parts; q0 += kBatch) {
+        float2 ml[kBatch];
+        float4 x[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            if (q0 + u < n_parts) {
+                const int slot = (q0 + u == 0) ? slot0 : 2 * (c0 + q0 + u);
+                ml[u] = *reinterpret_cast<const float2*>(pm + slot * (2 * kRows));
+                x[u] = *reinterpret_cast<const float4*>(po + slot * sstride);
+            } else {
+                ml[u] = make_float2(-INFINITY, 0.f);
+            }
+        }
+        float bm = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) bm = fmaxf(bm, ml[u].x);
+        const float nmx = fmaxf(mx, bm);
+        if (nmx == -INFINITY) continue;
+        const float sc = (mx == -INFINITY) ? 0.f : exp2f(mx - nmx);
+        den *= sc;
+        acc.x *= sc; acc.y *= sc; acc.z *= sc; acc.w *= sc;
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            if (ml[u].x == -INFINITY) continue;
+            const float w = exp2f(ml[u].x - nmx);
+            den += w * ml[u].y;
+            acc.x += w * x[u].x; acc.y += w * x[u].y; acc.z += w * x[u].z; acc.w += w * x[u].w;
+        }
+        mx = nmx;
+    }
+    const float inv = den > 0.f ? 1.f / den : 0.f;
+    *reinterpret_cast<uint2*>(o) = make_uint2(f2_to_bf2(acc.x * inv, acc.y * inv), f2_to_bf2(acc.z * inv, acc.w * inv));
+}
+
 // grid (n_split_tiles, kRows * D / 32 / kCombineThreads): the x-th query
 // tile that several attention blocks share.  Block cb = split_cb[x] is the
 // first to start inside the tile, so its partials are in the slots of blocks
@@ -176,7 +257,7 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
 // and merges the partials online, two at a time: both (max, sum) pairs
 // first, then each part's eight 4-column pieces.
 constexpr int kCombineThreads = 128;
-__global__ void __launch_bounds__(kCombineThreads) attn_combine_kernel(const __grid_constant__ AttnParams p) {
+__global__ void __launch_bounds__(kCombineThreads) attn_combine_group_kernel(const __grid_constant__ AttnParams p) {
     grid_dependency_wait();
     grid_dependents_launch();
     const int cb = p.split_cb[blockIdx.x];
@@ -301,8 +382,20 @@ void launch_rope_append(const AttnParams& p, int total_tokens, cudaStream_t s) {
 
 void launch_attn_combine(const AttnParams& p, cudaStream_t s) {
     if (p.n_split_tiles <= 0) return;
-    launch_pdl(attn_combine_kernel, dim3(p.n_split_tiles, (kRows * (p.D / 32) + kCombineThreads - 1) / kCombineThreads),
-               dim3(kCombineThreads), 0, s, p);
+    // one 4-column piece a thread while that grid is one wave (seven blocks
+    // an SM), else a 32-column group a thread: at npc (32 shared tiles) the
+    // piece form took 11.0 against 12.4 us, at long (128) 16.3 against 13.1
+    static int sms_of[64] = {};                      // per device
+    int dev = 0;
+    cudaGetDevice(&dev);
+    int& sms = sms_of[dev & 63];
+    if (!sms) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int piece_blocks = (kRows * (p.D / 4) + 255) / 256;
+    if ((int64_t)p.n_split_tiles * piece_blocks <= 7 * (int64_t)sms)
+        launch_pdl(attn_combine_piece_kernel, dim3(p.n_split_tiles, piece_blocks), dim3(256), 0, s, p);
+    else
+        launch_pdl(attn_combine_group_kernel, dim3(p.n_split_tiles, (kRows * (p.D / 32) + kCombineThreads - 1) / kCombineThreads),
+                   dim3(kCombineThreads), 0, s, p);
 }
 
 }  // namespace kvm
