@@ -14,7 +14,9 @@
 //  attn_combine : merge the partials of query tiles that the attention's
 //                persistent blocks split between them: each partial is an
 //                unnormalised accumulator with (reference max in log2 units,
-//                sum); one warp per query row.
+//                sum); a thread per 4-column piece of a row, or per 32-column
+//                group when the round shares more tiles than one wave of
+//                pieces covers.
 #include "kvm_internal.cuh"
 
 namespace kvm {
@@ -97,8 +99,9 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const __grid_constant_
                 if (rotated) lb[u] = *reinterpret_cast<const uint4*>(src + d0 + half);
             }
         }
-        // v needs no angle: copy it first
-        for (int idx = threadIdx.x; idx < p.Hkv * (D / 8); idx += blockDim.x) {
+        // v needs no angle: copy it first, from the block's last threads, so
+        // that the first ones form the angles meanwhile
+        for (int idx = blockDim.x - 1 - threadIdx.x; idx < p.Hkv * (D / 8); idx += blockDim.x) {
             const int h = idx / (D / 8), d0 = (idx % (D / 8)) * 8;
             *reinterpret_cast<uint4*>(p.V + ((int64_t)h * p.slab_rows + slot) * D + d0) =
                 *reinterpret_cast<const uint4*>(vrow + h * D + d0);
