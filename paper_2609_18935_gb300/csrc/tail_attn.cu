@@ -3,7 +3,7 @@
 //
 //  rope_append : rotate the tail's q and k at positions p + i, append the
 //                rotated k and v at live slots L' + i with their positions,
-//                and stage the rotated q for the attention's TMA loads.
+//                and write the rotated q for the attention's Q staging.
 //                The angle pos * omega_d is formed and reduced modulo 2*pi in
 //                fp64 (positions far beyond the live length stay accurate),
 //                then sin/cos and the rotation run in fp32.
